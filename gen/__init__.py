@@ -5,6 +5,8 @@ arithmetic the method performs on that data (no target softmax, nucleus
 filter, accept test, residual, top-k payload or branch selection).  Both the
 CUDA path's tests and the CPU oracle's tests read their inputs from here.
 """
-from .workloads import WORKLOADS, Workload, generate, generate_sequences, bf16_to_f32, f32_to_bf16
+from .workloads import (WORKLOADS, Workload, bf16_to_f32, f32_to_bf16, generate, generate_sequences,
+                        make_workload)
 
-__all__ = ["WORKLOADS", "Workload", "generate", "generate_sequences", "bf16_to_f32", "f32_to_bf16"]
+__all__ = ["WORKLOADS", "Workload", "generate", "generate_sequences", "make_workload", "bf16_to_f32",
+           "f32_to_bf16"]

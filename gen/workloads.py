@@ -136,10 +136,22 @@ def _one_sequence(w: Workload, b: int, head):
     return z32, q, xt, u
 
 
+def make_workload(B: int, K: int, V: int, dtype: str = "bf16", sigma: float = 3.0,
+                  rho: Optional[float] = 0.8, noise: float = 1.0, zipf: bool = False, T: float = 1.0,
+                  top_p: float = 0.9, k: int = 16, F: Sequence[int] = (), seed: int = 7,
+                  name: str = "custom") -> Workload:
+    """An ad-hoc workload with the same recipe (for ragged and edge-case tests)."""
+    F = tuple(F) if F else (2,) * K
+    return Workload(name, B, K, V, dtype, sigma, rho, noise, zipf, T, top_p, k, F, seed)
+
+
+def _resolve(w) -> Workload:
+    return WORKLOADS[w] if isinstance(w, str) else w
+
+
 def _fill(args):
-    name, seqs, shm_names, shapes = args
+    w, seqs, shm_names, shapes = args
     from multiprocessing import shared_memory
-    w = WORKLOADS[name]
     head = _zipf_head(w) if w.zipf else None
     shms = [shared_memory.SharedMemory(name=s) for s in shm_names]
     try:
@@ -160,14 +172,14 @@ def _fill(args):
     return len(seqs)
 
 
-def generate_sequences(name: str, seqs: Sequence[int], workers: int = 0, B: Optional[int] = None):
-    """Generate the listed sequences of workload `name`.
+def generate_sequences(name, seqs: Sequence[int], workers: int = 0, B: Optional[int] = None):
+    """Generate the listed sequences of workload `name` (a name or a Workload).
 
     Returns a dict with z ([n,K+1,V] float32, or uint16 bfloat16 bits), q
     ([n,K,V] float32), xt ([n,K] int32), u ([n,K+1] float32) and the workload.
     `workers` > 1 uses a spawn-started process pool (safe after CUDA init).
     """
-    w = WORKLOADS[name]
+    w = _resolve(name)
     seqs = [int(s) for s in seqs]
     n = len(seqs)
     zdt = np.uint16 if w.dtype == "bf16" else np.float32
@@ -191,7 +203,7 @@ def generate_sequences(name: str, seqs: Sequence[int], workers: int = 0, B: Opti
         chunks = [items[i::workers] for i in range(workers)]
         ctx = mp.get_context("spawn")
         with ctx.Pool(workers) as pool:
-            pool.map(_fill, [(name, c, [s.name for s in shms], shapes) for c in chunks if c])
+            pool.map(_fill, [(w, c, [s.name for s in shms], shapes) for c in chunks if c])
         out = [np.ndarray(s, dtype=d, buffer=m.buf).copy() for (s, d), m in zip(shapes, shms)]
     finally:
         for m in shms:
@@ -200,10 +212,10 @@ def generate_sequences(name: str, seqs: Sequence[int], workers: int = 0, B: Opti
     return dict(z=out[0], q=out[1], xt=out[2], u=out[3], w=w, seqs=np.array(seqs))
 
 
-def generate(name: str, workers: int = 0, B: Optional[int] = None):
+def generate(name, workers: int = 0, B: Optional[int] = None):
     """Generate the first B (default: all) sequences of workload `name`."""
-    w = WORKLOADS[name]
+    w = _resolve(name)
     nb = w.B if B is None else B
     if workers == 0:
         workers = min(16, os.cpu_count() or 1) if w.V * w.K * nb > 50_000_000 else 1
-    return generate_sequences(name, range(nb), workers=workers)
+    return generate_sequences(w, range(nb), workers=workers)

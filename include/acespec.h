@@ -1,0 +1,170 @@
+/*
+ * acespec.h -- C ABI of the AceSpec verify / sparsify / state-cache path on
+ * one GB300 GPU (sm_103a).
+ *
+ * AceSpec (arXiv 2609.02514) splits speculative decoding between an edge
+ * device and a cloud server.  The cloud verifies a drafted main chain of K
+ * tokens against the target model and answers with the first-rejection index
+ * pi and a sparse target distribution (Sec. III-B); the edge turns a
+ * rejection into an O(1) lookup in a probabilistic cache of alternative
+ * branches built per draft depth (Sec. III-C, Algorithm 1).  This library
+ * implements the vocabulary-wide per-position arithmetic of those steps.
+ * Verification follows the modified rejection sampling the paper relies on
+ * (Sec. II-A, Chen et al.), whose output has exactly the target distribution.
+ *
+ * Conventions shared by every entry point
+ *   - All array arguments are DEVICE pointers owned by the caller; the
+ *     library never allocates, frees or retains them.  F_host is the one
+ *     host array.
+ *   - Work is enqueued on `stream` and the call returns before it finishes.
+ *     A call returns ACES_OK once its kernels are launched.
+ *   - Arguments are validated before anything is launched; on
+ *     ACES_ERR_INVALID_ARG / ACES_ERR_UNSUPPORTED nothing is enqueued and no
+ *     output is touched.  ACES_ERR_CUDA reports a failed launch.
+ *   - Layouts are dense row-major with the vocabulary (V) contiguous.
+ *     Row r = b * (K + 1) + i addresses position i of sequence b.
+ *   - Order of a distribution: ids by (logit desc, id asc); exactly equal
+ *     logits are ordered by the lower id.  -0.0 equals +0.0.
+ *   - Data errors never trap: they are reported per row in row_status.
+ *
+ * Reading of points the paper leaves open (the library's contract):
+ *   - nucleus: the shortest prefix of the order whose softmax(z/T) mass
+ *     reaches top_p (the crossing id is kept); top_p = 1 keeps every id
+ *     with a finite logit; p is renormalised over the kept set.
+ *   - accept: a_i = [u_i < min(1, p_i(x~_i) / q_i(x~_i))]; q_i(x~_i) <= 0,
+ *     NaN, or an out-of-range draft token forces a reject (ACES_ROW_BAD_Q).
+ *   - pi_b = first i with a_i = 0, else K.  When pi < K the emitted token is
+ *     drawn from norm(max(0, p_pi - q_pi)) (from p_pi if that is all zero);
+ *     when pi = K the bonus token is drawn from p_K.  The draw is the
+ *     smallest id j whose prefix sum over ids 0..j exceeds u[b, K] times the
+ *     total.
+ *   - -inf logits are allowed (probability 0).  NaN or +inf logits, or a row
+ *     whose logits are all -inf, mark the row ACES_ROW_NONFINITE.
+ */
+#ifndef ACESPEC_H
+#define ACESPEC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    ACES_OK = 0,
+    ACES_ERR_INVALID_ARG = 1,
+    ACES_ERR_UNSUPPORTED = 2,
+    ACES_ERR_CUDA = 3
+} aces_status;
+
+typedef enum { ACES_F32 = 0, ACES_BF16 = 1 } aces_dtype;
+
+/* bits of row_status */
+#define ACES_ROW_NONFINITE 1 /* NaN / +inf logits, or all logits -inf      */
+#define ACES_ROW_BAD_Q 2     /* invalid draft probability or draft token   */
+
+/* The CUDA runtime's cudaStream_t (NULL = legacy default stream). */
+typedef struct CUstream_st *aces_stream_t;
+
+/* Limits checked by every entry point. */
+#define ACES_MAX_K 16        /* draft length gamma                        */
+#define ACES_MAX_V (1 << 20) /* vocabulary                                */
+#define ACES_MAX_TOPK 256    /* payload entries per row                   */
+#define ACES_MAX_BRANCH 1024 /* branches per depth                        */
+
+/*
+ * Bytes of device scratch that aces_verify (B sequences, K >= 1) or
+ * aces_sparsify (B rows, K = 0) needs.  The caller allocates it, passes it
+ * to the call and must not use it while the call's work is in flight; it
+ * needs no initialisation.  Returns 0 for invalid sizes.
+ */
+size_t aces_workspace_bytes(int B, int K, int V, int k);
+
+/*
+ * Cloud-side lossless verification of B drafted chains, fused with the
+ * sparse downlink payload (Sec. III-B; Algorithm 1 RECEIVE_WAIT / RESAMPLE
+ * inputs; Sec. V-C for the compact payload).
+ *
+ *   target_logits [B, K+1, V]  float32 or bfloat16 (dt); row K is the bonus
+ *                              position after the last draft token
+ *   draft_probs   [B, K, V]    float32, the edge model's distributions Q
+ *   draft_tokens  [B, K]       int32, the uploaded main chain x~
+ *   uniforms      [B, K+1]     float32 in (0,1); u[:, i<K] drive the accept
+ *                              tests, u[:, K] the single residual/bonus draw
+ *   T > 0, 0 < top_p <= 1      temperature and nucleus mass
+ * Outputs:
+ *   accept_len    [B]  int32   pi_b, accepted draft tokens (0..K)
+ *   out_token     [B]  int32   corrected (pi < K) or bonus (pi = K) token;
+ *                              -1 when that row is NONFINITE or its draft
+ *                              row holds NaN / negative probabilities
+ *   row_status    [B, K+1]     int32 ACES_ROW_* bits per row
+ * Sparse payload (k >= 1; k = 0 skips it and the three pointers may be NULL):
+ *   topk_ids      [B, K+1, k]  int32   first k ids of every row's nucleus
+ *                              in order, -1 padding
+ *   topk_probs    [B, K+1, k]  float32 their renormalised p, 0 padding
+ *   tail_mass     [B, K+1]     float32 1 - sum of the row's topk_probs
+ * workspace / workspace_bytes: device scratch of at least
+ *   aces_workspace_bytes(B, K, V, k) bytes, 16-byte aligned.
+ * Limits: 1 <= B, 1 <= K <= ACES_MAX_K, 2 <= V <= ACES_MAX_V,
+ *   0 <= k <= min(V, ACES_MAX_TOPK).
+ */
+aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                        const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                        float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                        int32_t *topk_ids, float *topk_probs, float *tail_mass,
+                        int32_t *row_status, void *workspace, size_t workspace_bytes,
+                        aces_stream_t stream);
+
+/*
+ * Sparse payload alone for `rows` independent target rows (the COMPRESS of
+ * the downlink distribution, Sec. III-B and Sec. V-C): temperature softmax,
+ * nucleus, then the first k ids of the nucleus with their renormalised
+ * probabilities and the tail mass.
+ *   target_logits [rows, V]; outputs topk_ids / topk_probs [rows, k],
+ *   tail_mass [rows], row_status [rows].
+ * workspace: at least aces_workspace_bytes(rows, 0, V, k) bytes.
+ * Limits: rows >= 1, 2 <= V <= ACES_MAX_V, 1 <= k <= min(V, ACES_MAX_TOPK).
+ */
+aces_status aces_sparsify(const void *target_logits, aces_dtype dt, int rows, int V, float T,
+                          float top_p, int k, int32_t *topk_ids, float *topk_probs,
+                          float *tail_mass, int32_t *row_status, void *workspace,
+                          size_t workspace_bytes, aces_stream_t stream);
+
+/*
+ * Edge-side probabilistic state cache (Sec. III-C; Algorithm 1 TREE_DRAFT):
+ * at every draft depth d < K, the F_d most probable alternative tokens of
+ * the draft distribution q[b, d, :] other than the main-chain token
+ * x~[b, d], ordered by (q desc, id asc), among ids with q > 0, with branch
+ * probability q(x) / (1 - q(x~[b, d])).
+ *   draft_probs  [B, K, V] float32, draft_tokens [B, K] int32
+ *   F_host       [K] host int32 fan-out vector (Sec. IV-B), 0 <= F_d <=
+ *                min(V - 1, ACES_MAX_BRANCH)
+ * Outputs, S = sum F:  branch_tok [B, S] int32 (-1 padding when fewer ids
+ *   qualify, or when 1 - q(x~) <= 0 or x~ is out of range),
+ *   branch_prob [B, S] float32 (0 padding).  Depth d occupies columns
+ *   [off_d, off_d + F_d) with off_d = F_0 + ... + F_{d-1}.
+ */
+aces_status aces_cache_build(const float *draft_probs, const int32_t *draft_tokens,
+                             const int32_t *F_host, int B, int K, int V, int32_t *branch_tok,
+                             float *branch_prob, aces_stream_t stream);
+
+/*
+ * O(1) state recovery lookup (Sec. III-B, Algorithm 1: w = (pi, x_resampled),
+ * w in dom(T)).  For each sequence: slot[b] = off_pi + j when
+ * branch_tok[b, off_pi + j] == token[b] (the first such j); -1 on a miss or
+ * when token[b] < 0; -2 when accept_len[b] == K (the whole chain was
+ * accepted and the main chain continues).
+ *   branch_tok [B, sum F], accept_len [B], token [B] -> slot [B] (int32).
+ */
+aces_status aces_cache_lookup(const int32_t *branch_tok, const int32_t *F_host, int B, int K,
+                              const int32_t *accept_len, const int32_t *token, int32_t *slot,
+                              aces_stream_t stream);
+
+/* Static English text for a status code. */
+const char *aces_status_string(aces_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ACESPEC_H */

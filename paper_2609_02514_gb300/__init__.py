@@ -1,0 +1,211 @@
+"""AceSpec verify / sparsify / state-cache path on one GB300 GPU.
+
+Thin Python binding of libacespec.so (declared in include/acespec.h).  The
+functions below only marshal arguments: output tensors are allocated with
+PyTorch on the inputs' device, pointers and the current CUDA stream are
+handed to the C ABI, and every step of the computation runs in the
+library's CUDA kernels.  There is no CPU fallback: calling any function
+without the built library, or with host tensors, raises.
+
+    verify(z, q, xt, u, T, top_p, k)      Sec. III-B, lossless verification
+                                          fused with the sparse payload
+    sparsify(z, T, top_p, k)              Sec. III-B / V-C downlink payload
+    cache_build(q, xt, F)                 Sec. III-C branch cache
+    cache_lookup(branch_tok, F, pi, tok)  Algorithm 1 state recovery
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+__all__ = ["load", "lib_path", "workspace_bytes", "verify", "sparsify", "cache_build", "cache_lookup",
+           "ROW_NONFINITE", "ROW_BAD_Q", "AcespecError"]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "libacespec.so")
+_lock = threading.Lock()
+_lib = None
+
+ROW_NONFINITE = 1
+ROW_BAD_Q = 2
+ACES_F32 = 0
+ACES_BF16 = 1
+_STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported argument", 3: "CUDA launch error"}
+
+
+class AcespecError(RuntimeError):
+    def __init__(self, fn, code):
+        super().__init__(f"{fn} failed: {_STATUS.get(code, code)} (status {code})")
+        self.code = code
+
+
+def lib_path() -> str:
+    return _LIB_PATH
+
+
+def load():
+    """Load libacespec.so (built by __graft_entry__.build() or build.py)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(f"{_LIB_PATH} is missing: build it with `python -m paper_2609_02514_gb300.build`")
+        lib = ctypes.CDLL(_LIB_PATH)
+        P, I, F, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+        lib.aces_workspace_bytes.argtypes = [I, I, I, I]
+        lib.aces_workspace_bytes.restype = S
+        lib.aces_verify.argtypes = [P, I, P, P, P, I, I, I, F, F, P, P, I, P, P, P, P, P, S, P]
+        lib.aces_sparsify.argtypes = [P, I, I, I, F, F, I, P, P, P, P, P, S, P]
+        lib.aces_cache_build.argtypes = [P, P, P, I, I, I, P, P, P]
+        lib.aces_cache_lookup.argtypes = [P, P, I, I, P, P, P, P]
+        lib.aces_status_string.argtypes = [I]
+        lib.aces_status_string.restype = ctypes.c_char_p
+        for f in (lib.aces_verify, lib.aces_sparsify, lib.aces_cache_build, lib.aces_cache_lookup):
+            f.restype = I
+        _lib = lib
+        return lib
+
+
+def _check(fn, code):
+    if code != 0:
+        raise AcespecError(fn, code)
+
+
+def _cuda(t: torch.Tensor, name: str) -> torch.Tensor:
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(dev):
+    return ctypes.c_void_p(torch.cuda.current_stream(dev).cuda_stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return ACES_F32
+    if t.dtype == torch.bfloat16:
+        return ACES_BF16
+    raise ValueError(f"target logits must be float32 or bfloat16, got {t.dtype}")
+
+
+def workspace_bytes(B: int, K: int, V: int, k: int) -> int:
+    return int(load().aces_workspace_bytes(int(B), int(K), int(V), int(k)))
+
+
+def verify(target_logits, draft_probs, draft_tokens, uniforms, T: float, top_p: float, k: int = 0,
+           out: dict | None = None, workspace: torch.Tensor | None = None):
+    """Lossless verification of B drafted chains (+ sparse payload when k > 0).
+
+    target_logits [B, K+1, V] float32/bfloat16, draft_probs [B, K, V] float32,
+    draft_tokens [B, K] int32, uniforms [B, K+1] float32.
+    Returns a dict of device tensors: accept_len [B], out_token [B],
+    row_status [B, K+1] and, when k > 0, topk_ids / topk_probs [B, K+1, k],
+    tail_mass [B, K+1].  `out` may supply preallocated outputs (same keys).
+    """
+    lib = load()
+    z = _cuda(target_logits, "target_logits")
+    q = _cuda(draft_probs, "draft_probs")
+    xt = _cuda(draft_tokens, "draft_tokens")
+    u = _cuda(uniforms, "uniforms")
+    if z.dim() != 3:
+        raise ValueError("target_logits must be [B, K+1, V]")
+    B, R, V = z.shape
+    K = R - 1
+    if q.dtype != torch.float32 or tuple(q.shape) != (B, K, V):
+        raise ValueError("draft_probs must be float32 [B, K, V]")
+    if xt.dtype != torch.int32 or tuple(xt.shape) != (B, K):
+        raise ValueError("draft_tokens must be int32 [B, K]")
+    if u.dtype != torch.float32 or tuple(u.shape) != (B, R):
+        raise ValueError("uniforms must be float32 [B, K+1]")
+    dev = z.device
+    o = {} if out is None else dict(out)
+    i32 = dict(dtype=torch.int32, device=dev)
+    f32 = dict(dtype=torch.float32, device=dev)
+    o.setdefault("accept_len", torch.empty(B, **i32))
+    o.setdefault("out_token", torch.empty(B, **i32))
+    o.setdefault("row_status", torch.empty(B, R, **i32))
+    if k > 0:
+        o.setdefault("topk_ids", torch.empty(B, R, k, **i32))
+        o.setdefault("topk_probs", torch.empty(B, R, k, **f32))
+        o.setdefault("tail_mass", torch.empty(B, R, **f32))
+    need = workspace_bytes(B, K, V, k)
+    ws = workspace if workspace is not None else torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    code = lib.aces_verify(_p(z), _dtype_code(z), _p(q), _p(xt), _p(u), B, K, V, float(T), float(top_p),
+                           _p(o["accept_len"]), _p(o["out_token"]), int(k), _p(o.get("topk_ids")),
+                           _p(o.get("topk_probs")), _p(o.get("tail_mass")), _p(o["row_status"]),
+                           _p(ws), ws.numel(), _stream(dev))
+    _check("aces_verify", code)
+    return o
+
+
+def sparsify(target_logits, T: float, top_p: float, k: int, out: dict | None = None,
+             workspace: torch.Tensor | None = None):
+    """Sparse top-k payload of every row of target_logits [rows, V] (or [..., V])."""
+    lib = load()
+    z = _cuda(target_logits, "target_logits")
+    V = z.shape[-1]
+    rows = z.numel() // V
+    dev = z.device
+    lead = tuple(z.shape[:-1])
+    o = {} if out is None else dict(out)
+    o.setdefault("topk_ids", torch.empty(*lead, k, dtype=torch.int32, device=dev))
+    o.setdefault("topk_probs", torch.empty(*lead, k, dtype=torch.float32, device=dev))
+    o.setdefault("tail_mass", torch.empty(*lead, dtype=torch.float32, device=dev))
+    o.setdefault("row_status", torch.empty(*lead, dtype=torch.int32, device=dev))
+    need = workspace_bytes(rows, 0, V, k)
+    ws = workspace if workspace is not None else torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    code = lib.aces_sparsify(_p(z), _dtype_code(z), rows, V, float(T), float(top_p), int(k),
+                             _p(o["topk_ids"]), _p(o["topk_probs"]), _p(o["tail_mass"]),
+                             _p(o["row_status"]), _p(ws), ws.numel(), _stream(dev))
+    _check("aces_sparsify", code)
+    return o
+
+
+def _f_host(F):
+    arr = (ctypes.c_int32 * len(F))(*[int(f) for f in F])
+    return arr
+
+
+def cache_build(draft_probs, draft_tokens, F, out: dict | None = None):
+    """Branch cache: q [B,K,V] float32, x~ [B,K] int32, F (K ints) ->
+    branch_tok [B, sum F] int32, branch_prob [B, sum F] float32."""
+    lib = load()
+    q = _cuda(draft_probs, "draft_probs")
+    xt = _cuda(draft_tokens, "draft_tokens")
+    B, K, V = q.shape
+    if len(F) != K:
+        raise ValueError("F must have K entries")
+    tot = int(sum(int(f) for f in F))
+    dev = q.device
+    o = {} if out is None else dict(out)
+    o.setdefault("branch_tok", torch.empty(B, tot, dtype=torch.int32, device=dev))
+    o.setdefault("branch_prob", torch.empty(B, tot, dtype=torch.float32, device=dev))
+    code = lib.aces_cache_build(_p(q), _p(xt), _f_host(F), B, K, V, _p(o["branch_tok"]),
+                                _p(o["branch_prob"]), _stream(dev))
+    _check("aces_cache_build", code)
+    return o
+
+
+def cache_lookup(branch_tok, F, accept_len, token, out: torch.Tensor | None = None):
+    """slot [B] int32: off_pi + j on a hit, -1 on a miss, -2 when pi == K."""
+    lib = load()
+    bt = _cuda(branch_tok, "branch_tok")
+    al = _cuda(accept_len, "accept_len")
+    tk = _cuda(token, "token")
+    B = al.shape[0]
+    K = len(F)
+    slot = out if out is not None else torch.empty(B, dtype=torch.int32, device=al.device)
+    code = lib.aces_cache_lookup(_p(bt), _f_host(F), B, K, _p(al), _p(tk), _p(slot), _stream(al.device))
+    _check("aces_cache_lookup", code)
+    return slot

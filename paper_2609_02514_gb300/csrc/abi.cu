@@ -1,0 +1,243 @@
+// C ABI of the AceSpec path: argument validation, launch configuration and
+// workspace carving.  Nothing here allocates memory.
+#include <climits>
+#include <cmath>
+
+#include "common.cuh"
+
+using namespace aces;
+
+namespace {
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 132;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 132;
+    return n;
+}
+
+size_t elem_size(aces_dtype dt) { return dt == ACES_BF16 ? 2 : 4; }
+
+// Common checks of the target-row arguments.  Returns ACES_OK or the error.
+aces_status check_rows(const void *logits, aces_dtype dt, long long rows, int V, float T, float top_p,
+                       int k, bool need_payload, const void *ids, const void *probs, const void *tail,
+                       const void *status) {
+    if (dt != ACES_F32 && dt != ACES_BF16) return ACES_ERR_UNSUPPORTED;
+    if (!logits || !status) return ACES_ERR_INVALID_ARG;
+    if (rows < 1 || rows > INT_MAX / 2) return ACES_ERR_INVALID_ARG;
+    if (V < 2 || V > ACES_MAX_V) return ACES_ERR_INVALID_ARG;
+    if (T == 0.0f) return ACES_ERR_UNSUPPORTED;  // greedy decoding is not a distribution
+    if (!(T > 0.0f) || !std::isfinite(T)) return ACES_ERR_INVALID_ARG;
+    if (!(top_p > 0.0f && top_p <= 1.0f)) return ACES_ERR_INVALID_ARG;
+    if (k < 0 || k > ACES_MAX_TOPK || k > V) return ACES_ERR_INVALID_ARG;
+    if (need_payload && k < 1) return ACES_ERR_INVALID_ARG;
+    if (k > 0 && (!ids || !probs || !tail)) return ACES_ERR_INVALID_ARG;
+    (void)elem_size;
+    return ACES_OK;
+}
+
+// Row kernels: fast sketch path when rows are 16-byte aligned, then the
+// exact general path for every row the fast path handed over.
+aces_status run_rows(RowArgs &a, aces_dtype dt, cudaStream_t s) {
+    const size_t es = elem_size(dt);
+    const bool vec = aligned16(a.logits) && ((size_t)a.V * es) % 16 == 0;
+    const int nsm = sm_count();
+    if (cudaMemsetAsync(a.ws.fb_count, 0, 16, s) != cudaSuccess) return ACES_ERR_CUDA;
+    if (vec) {
+        const int epc = dt == ACES_BF16 ? 8 : 4;
+        const int nch = a.V / epc;
+        const int gmax = dt == ACES_BF16 ? 8 : 16;
+        int gc = 2;
+        while (gc < gmax && (nch + gc - 1) / gc > SKETCH_CAP) gc *= 2;
+        a.ng = (nch + gc - 1) / gc;
+        const size_t smem = align16((size_t)a.ng * 4) + (size_t)CAND_CAP * 8;
+        if (launch_rows_fast(a, dt, gc, smem, s) != cudaSuccess) return ACES_ERR_CUDA;
+        int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
+        if (launch_rows_general(a, dt, true, 0, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
+    } else {
+        a.ng = 0;
+        int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
+        if (launch_rows_general(a, dt, false, 1, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
+    }
+    return ACES_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t aces_workspace_bytes(int B, int K, int V, int k) {
+    if (B < 1 || K < 0 || K > ACES_MAX_K || V < 2 || V > ACES_MAX_V || k < 0 || k > ACES_MAX_TOPK)
+        return 0;
+    long long rows = (long long)B * (K + 1);
+    if (rows > INT_MAX / 2) return 0;
+    return ws_bytes((int)rows, B * K);
+}
+
+aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                        const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                        float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                        int32_t *topk_ids, float *topk_probs, float *tail_mass,
+                        int32_t *row_status, void *workspace, size_t workspace_bytes,
+                        aces_stream_t stream) {
+    if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
+    aces_status st = check_rows(target_logits, dt, (long long)B * (K + 1), V, T, top_p, k, false,
+                                topk_ids, topk_probs, tail_mass, row_status);
+    if (st != ACES_OK) return st;
+    if (!draft_probs || !draft_tokens || !uniforms || !accept_len || !out_token || !workspace)
+        return ACES_ERR_INVALID_ARG;
+    if (!aligned16(workspace) || workspace_bytes < aces_workspace_bytes(B, K, V, k))
+        return ACES_ERR_INVALID_ARG;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const int rows = B * (K + 1);
+    RowArgs a;
+    a.logits = target_logits;
+    a.rows = rows;
+    a.V = V;
+    a.K = K;
+    a.T = T;
+    a.c = (float)(1.4426950408889634 / (double)T);
+    a.inv_w = (float)(BIN_PER_T / (double)T);
+    a.top_p = top_p;
+    a.k = k;
+    a.q = draft_probs;
+    a.xt = draft_tokens;
+    a.u = uniforms;
+    a.topk_ids = topk_ids;
+    a.topk_probs = topk_probs;
+    a.tail = tail_mass;
+    a.row_status = row_status;
+    a.ws = ws_carve(workspace, rows, B * K);
+    a.ng = 0;
+    st = run_rows(a, dt, s);
+    if (st != ACES_OK) return st;
+    ResolveArgs r;
+    r.logits = target_logits;
+    r.q = draft_probs;
+    r.u = uniforms;
+    r.B = B;
+    r.K = K;
+    r.V = V;
+    r.ws = a.ws;
+    r.accept_len = accept_len;
+    r.out_token = out_token;
+    r.row_status = row_status;
+    const bool vec = aligned16(target_logits) && ((size_t)V * elem_size(dt)) % 16 == 0 &&
+                     aligned16(draft_probs) && V % 4 == 0;
+    if (launch_resolve(r, dt, vec, s) != cudaSuccess) return ACES_ERR_CUDA;
+    return ACES_OK;
+}
+
+aces_status aces_sparsify(const void *target_logits, aces_dtype dt, int rows, int V, float T,
+                          float top_p, int k, int32_t *topk_ids, float *topk_probs,
+                          float *tail_mass, int32_t *row_status, void *workspace,
+                          size_t workspace_bytes, aces_stream_t stream) {
+    aces_status st = check_rows(target_logits, dt, rows, V, T, top_p, k, true, topk_ids, topk_probs,
+                                tail_mass, row_status);
+    if (st != ACES_OK) return st;
+    if (!workspace || !aligned16(workspace) || workspace_bytes < aces_workspace_bytes(rows, 0, V, k))
+        return ACES_ERR_INVALID_ARG;
+    RowArgs a;
+    a.logits = target_logits;
+    a.rows = rows;
+    a.V = V;
+    a.K = 0;
+    a.T = T;
+    a.c = (float)(1.4426950408889634 / (double)T);
+    a.inv_w = (float)(BIN_PER_T / (double)T);
+    a.top_p = top_p;
+    a.k = k;
+    a.q = nullptr;
+    a.xt = nullptr;
+    a.u = nullptr;
+    a.topk_ids = topk_ids;
+    a.topk_probs = topk_probs;
+    a.tail = tail_mass;
+    a.row_status = row_status;
+    a.ws = ws_carve(workspace, rows, 0);
+    a.ng = 0;
+    return run_rows(a, dt, reinterpret_cast<cudaStream_t>(stream));
+}
+
+static aces_status fill_cache_args(CacheArgs &c, const int32_t *F_host, int B, int K, int V) {
+    if (!F_host || B < 1 || K < 1 || K > ACES_MAX_K || V < 2 || V > ACES_MAX_V) return ACES_ERR_INVALID_ARG;
+    if ((long long)B * K > INT_MAX / 2) return ACES_ERR_INVALID_ARG;
+    int tot = 0;
+    c.off[0] = 0;
+    for (int d = 0; d < K; ++d) {
+        int f = F_host[d];
+        if (f < 0 || f > V - 1) return ACES_ERR_INVALID_ARG;
+        if (f > ACES_MAX_BRANCH) return ACES_ERR_UNSUPPORTED;
+        c.F[d] = f;
+        tot += f;
+        c.off[d + 1] = tot;
+    }
+    for (int d = K; d < ACES_MAX_K; ++d) c.F[d] = 0;
+    c.total = tot;
+    c.B = B;
+    c.K = K;
+    c.V = V;
+    return ACES_OK;
+}
+
+aces_status aces_cache_build(const float *draft_probs, const int32_t *draft_tokens,
+                             const int32_t *F_host, int B, int K, int V, int32_t *branch_tok,
+                             float *branch_prob, aces_stream_t stream) {
+    CacheArgs c;
+    aces_status st = fill_cache_args(c, F_host, B, K, V);
+    if (st != ACES_OK) return st;
+    if (!draft_probs || !draft_tokens) return ACES_ERR_INVALID_ARG;
+    if (c.total == 0) return ACES_OK;
+    if (!branch_tok || !branch_prob) return ACES_ERR_INVALID_ARG;
+    c.q = draft_probs;
+    c.xt = draft_tokens;
+    c.bt = branch_tok;
+    c.bp = branch_prob;
+    const bool vec = aligned16(draft_probs) && V % 4 == 0;
+    if (launch_cache_build(c, vec, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return ACES_ERR_CUDA;
+    return ACES_OK;
+}
+
+aces_status aces_cache_lookup(const int32_t *branch_tok, const int32_t *F_host, int B, int K,
+                              const int32_t *accept_len, const int32_t *token, int32_t *slot,
+                              aces_stream_t stream) {
+    CacheArgs c;
+    if (!F_host || B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
+    int tot = 0;
+    c.off[0] = 0;
+    for (int d = 0; d < K; ++d) {
+        if (F_host[d] < 0 || F_host[d] > ACES_MAX_BRANCH) return ACES_ERR_INVALID_ARG;
+        c.F[d] = F_host[d];
+        tot += F_host[d];
+        c.off[d + 1] = tot;
+    }
+    for (int d = K; d < ACES_MAX_K; ++d) c.F[d] = 0;
+    c.total = tot;
+    c.B = B;
+    c.K = K;
+    c.V = 0;
+    c.q = nullptr;
+    c.xt = nullptr;
+    c.bt = nullptr;
+    c.bp = nullptr;
+    if (!accept_len || !token || !slot || (tot > 0 && !branch_tok)) return ACES_ERR_INVALID_ARG;
+    if (launch_cache_lookup(branch_tok, c, accept_len, token, slot,
+                            reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return ACES_ERR_CUDA;
+    return ACES_OK;
+}
+
+const char *aces_status_string(aces_status s) {
+    switch (s) {
+        case ACES_OK: return "ok";
+        case ACES_ERR_INVALID_ARG: return "invalid argument";
+        case ACES_ERR_UNSUPPORTED: return "unsupported argument";
+        case ACES_ERR_CUDA: return "CUDA launch error";
+    }
+    return "unknown status";
+}
+
+}  // extern "C"

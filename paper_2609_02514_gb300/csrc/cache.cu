@@ -1,0 +1,139 @@
+// Probabilistic state cache of the AceSpec edge step (Sec. III-C,
+// Algorithm 1 TREE_DRAFT and the O(1) lookup of w = (pi, x_resampled)).
+//
+//   k_cache_build   one CTA per (sequence, depth) row of the draft
+//                   distribution: the F_d largest q over ids != x~_d, in
+//                   (q desc, id asc) order, with probability q / (1 - q(x~_d)).
+//                   One HBM pass keeps a sorted top-8 list per thread; the
+//                   block then extracts maxima one at a time.  Fan-outs above
+//                   8 repeat the pass below the last extracted order value.
+//   k_cache_lookup  one thread per sequence scanning the F_pi branches.
+#include "common.cuh"
+
+namespace aces {
+
+
+constexpr int TOPL = 8;  // per-thread list length
+
+__device__ __forceinline__ void list_insert(unsigned long long (&Lst)[TOPL], unsigned long long o) {
+    if (o > Lst[TOPL - 1]) {
+        Lst[TOPL - 1] = o;
+#pragma unroll
+        for (int i = TOPL - 1; i > 0; --i) {
+            if (Lst[i] > Lst[i - 1]) {
+                unsigned long long t = Lst[i];
+                Lst[i] = Lst[i - 1];
+                Lst[i - 1] = t;
+            }
+        }
+    }
+}
+
+template <bool VEC>
+__global__ void __launch_bounds__(NT) k_cache_build(CacheArgs a) {
+    __shared__ unsigned long long redu[NWARP];
+    const int row = blockIdx.x, tid = threadIdx.x;
+    const int b = row / a.K, d = row % a.K;
+    const int Fd = a.F[d];
+    if (Fd == 0) return;
+    const float *qr = a.q + (size_t)row * a.V;
+    int32_t *bt = a.bt + (size_t)b * a.total + a.off[d];
+    float *bp = a.bp + (size_t)b * a.total + a.off[d];
+    const int xd = a.xt[row];
+    float den = 0.0f;
+    if (xd >= 0 && xd < a.V) den = 1.0f - __ldg(qr + xd);
+    int got = 0;
+    if (den > 0.0f) {
+        unsigned long long ub = ~0ull;  // exclusive upper bound of this pass
+        while (got < Fd) {
+            unsigned long long Lst[TOPL];
+#pragma unroll
+            for (int i = 0; i < TOPL; ++i) Lst[i] = 0ull;
+            if (VEC) {
+                const int nch = a.V >> 2;
+#pragma unroll 4
+                for (int cc = tid; cc < nch; cc += NT) {
+                    uint4 w = ldg16(qr + (size_t)cc * 4);
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        float qv = Elem<ACES_F32>::get(w, e);
+                        int x = cc * 4 + e;
+                        if (qv > 0.0f && x != xd) {
+                            unsigned long long o = order_val(__float_as_uint(qv) | 0x80000000u, (uint32_t)x);
+                            if (o < ub) list_insert(Lst, o);
+                        }
+                    }
+                }
+            } else {
+                for (int x = tid; x < a.V; x += NT) {
+                    float qv = __ldg(qr + x);
+                    if (qv > 0.0f && x != xd) {
+                        unsigned long long o = order_val(__float_as_uint(qv) | 0x80000000u, (uint32_t)x);
+                        if (o < ub) list_insert(Lst, o);
+                    }
+                }
+            }
+            const int take = min(TOPL, Fd - got);
+            bool exhausted = false;
+            for (int t = 0; t < take; ++t) {
+                unsigned long long best = block_reduce(Lst[0], redu, MaxU64());
+                if (best == 0ull) {
+                    exhausted = true;
+                    break;
+                }
+                if (Lst[0] == best) {  // order values are unique: one owner
+#pragma unroll
+                    for (int i = 0; i < TOPL - 1; ++i) Lst[i] = Lst[i + 1];
+                    Lst[TOPL - 1] = 0ull;
+                }
+                if (tid == 0) {
+                    bt[got] = (int32_t)order_id(best);
+                    bp[got] = order_value(best) / den;
+                }
+                ++got;
+                ub = best;
+            }
+            if (exhausted) break;
+        }
+    }
+    for (int j = got + tid; j < Fd; j += NT) {
+        bt[j] = -1;
+        bp[j] = 0.0f;
+    }
+}
+
+__global__ void k_cache_lookup(const int32_t *bt, CacheArgs a, const int32_t *accept_len,
+                               const int32_t *token, int32_t *slot) {
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= a.B) return;
+    const int pi = accept_len[b];
+    if (pi == a.K) {
+        slot[b] = -2;
+        return;
+    }
+    int s = -1;
+    const int tok = token[b];
+    if (pi >= 0 && pi < a.K && tok >= 0) {
+        const int32_t *row = bt + (size_t)b * a.total + a.off[pi];
+        for (int j = 0; j < a.F[pi]; ++j)
+            if (row[j] == tok) {
+                s = a.off[pi] + j;
+                break;
+            }
+    }
+    slot[b] = s;
+}
+
+cudaError_t launch_cache_build(const CacheArgs &a, bool vec, cudaStream_t s) {
+    if (vec) k_cache_build<true><<<a.B * a.K, NT, 0, s>>>(a);
+    else k_cache_build<false><<<a.B * a.K, NT, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_cache_lookup(const int32_t *bt, const CacheArgs &a, const int32_t *accept_len,
+                                const int32_t *token, int32_t *slot, cudaStream_t s) {
+    k_cache_lookup<<<(a.B + 255) / 256, 256, 0, s>>>(bt, a, accept_len, token, slot);
+    return cudaGetLastError();
+}
+
+}  // namespace aces

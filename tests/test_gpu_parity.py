@@ -1,0 +1,253 @@
+"""Parity of the CUDA path (through the C ABI) with the float64 oracle.
+
+Every comparison uses the rules in tests/parity.py.  Inputs come from the
+seeded generator package only; a few edge-case tests then overwrite chosen
+entries of those inputs before handing the same arrays to both sides.
+"""
+import os
+
+import numpy as np
+import pytest
+
+import gen
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def A():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2609_02514_gb300 as A
+    A.load()
+    return A
+
+
+def _dev(inp):
+    z = inp["z"]
+    if z.dtype == np.uint16:
+        zt = torch.from_numpy(z.view(np.int16)).cuda().view(torch.bfloat16)
+    else:
+        zt = torch.from_numpy(z).cuda()
+    return (zt, torch.from_numpy(inp["q"]).cuda(), torch.from_numpy(inp["xt"]).cuda(),
+            torch.from_numpy(inp["u"]).cuda())
+
+
+def _np(d):
+    return {k: v.cpu().numpy() for k, v in d.items()}
+
+
+def run_gpu(A, inp, w, k):
+    z, q, xt, u = _dev(inp)
+    out = A.verify(z, q, xt, u, w.T, w.top_p, k)
+    torch.cuda.synchronize()
+    return _np(out)
+
+
+def run_gpu_cache(A, inp, F):
+    q = torch.from_numpy(inp["q"]).cuda()
+    xt = torch.from_numpy(inp["xt"]).cuda()
+    out = A.cache_build(q, xt, F)
+    torch.cuda.synchronize()
+    return out["branch_tok"].cpu().numpy(), out["branch_prob"].cpu().numpy()
+
+
+def check_all(A, orc, inp, w, k=None):
+    k = w.k if k is None else k
+    g = run_gpu(A, inp, w, k)
+    o = orc.verify(inp["z"], inp["q"], inp["xt"], inp["u"], w.T, w.top_p, k)
+    res = parity.compare_verify(inp, g, o, w.top_p, inp["z"].dtype == np.uint16, k)
+    return g, o, res
+
+
+def check_cache(A, orc, inp, F, g=None):
+    gbt, gbp = run_gpu_cache(A, inp, F)
+    obt, obp = orc.cache_build(inp["q"], inp["xt"], F)
+    parity.compare_cache(gbt, gbp, obt, obp)
+    if g is not None:
+        al = torch.from_numpy(g["accept_len"]).cuda()
+        tk = torch.from_numpy(g["out_token"]).cuda()
+        slot = A.cache_lookup(torch.from_numpy(gbt).cuda(), F, al, tk).cpu().numpy()
+        np.testing.assert_array_equal(slot, orc.cache_lookup(gbt, F, g["accept_len"], g["out_token"]))
+    return gbt
+
+
+# ---------------------------------------------------------------------------
+# the paper-shaped workloads
+
+
+@pytest.mark.parametrize("name", ["b1_k4_v32000_f32", "b16_k8_v32000_f32"])
+def test_small_workloads_full(A, orc, name):
+    inp = gen.generate(name)
+    w = inp["w"]
+    g, o, res = check_all(A, orc, inp, w)
+    assert res["checked_seqs"] >= w.B - 2
+    check_cache(A, orc, inp, w.F, g)
+
+
+@pytest.mark.parametrize("name", ["b64_k8_v152064_bf16", "b128_k16_v128256_bf16", "b256_k16_v256000_bf16"])
+def test_full_size_sampled(A, orc, name):
+    """Full batch on the GPU as the benchmark launches it; the oracle checks
+    sampled sequences one by one; properties are checked on every sequence."""
+    w = gen.WORKLOADS[name]
+    inp = gen.generate(name, workers=min(16, os.cpu_count() or 1))
+    g = run_gpu(A, inp, w, w.k)
+    B, K = w.B, w.K
+    # properties on all sequences
+    assert ((g["accept_len"] >= 0) & (g["accept_len"] <= K)).all()
+    assert ((g["out_token"] >= 0) & (g["out_token"] < w.V)).all()
+    rej = g["accept_len"] < K
+    xt_pi = inp["xt"][np.arange(B), np.minimum(g["accept_len"], K - 1)]
+    assert not np.any(g["out_token"][rej] == xt_pi[rej]), "a rejected draft token was re-emitted"
+    p = g["topk_probs"]
+    assert (np.diff(p, axis=-1) <= 1e-7).all(), "payload not in descending order"
+    assert (p.sum(-1) <= 1 + 1e-5).all()
+    np.testing.assert_allclose(g["tail_mass"], 1.0 - p.astype(np.float64).sum(-1), atol=2e-5)
+    assert (g["row_status"] == 0).all()
+    # oracle on a sample of sequences
+    rng = np.random.default_rng(5)
+    seqs = sorted(set([0, B - 1] + rng.choice(B, 4, replace=False).tolist()))
+    sub = {key: inp[key][seqs] for key in ("z", "q", "xt", "u")}
+    o = orc.verify(sub["z"], sub["q"], sub["xt"], sub["u"], w.T, w.top_p, w.k)
+    gs = {key: v[seqs] for key, v in g.items()}
+    res = parity.compare_verify(sub, gs, o, w.top_p, True, w.k)
+    assert res["checked_seqs"] >= len(seqs) - 2, res
+    # branch cache on the same sample
+    qt = torch.from_numpy(inp["q"]).cuda()
+    out = A.cache_build(qt, torch.from_numpy(inp["xt"]).cuda(), w.F)
+    del qt
+    gbt = out["branch_tok"].cpu().numpy()
+    gbp = out["branch_prob"].cpu().numpy()
+    obt, obp = orc.cache_build(sub["q"], sub["xt"], w.F)
+    parity.compare_cache(gbt[seqs], gbp[seqs], obt, obp)
+    slot = A.cache_lookup(out["branch_tok"], w.F, torch.from_numpy(g["accept_len"]).cuda(),
+                          torch.from_numpy(g["out_token"]).cuda()).cpu().numpy()
+    np.testing.assert_array_equal(slot, orc.cache_lookup(gbt, w.F, g["accept_len"], g["out_token"]))
+
+
+# ---------------------------------------------------------------------------
+# ragged sizes (several tiles plus a tail), both row paths
+
+
+RAGGED = [
+    dict(B=3, K=2, V=10007, dtype="f32", T=0.7, top_p=0.9, k=37),     # unaligned rows: general path
+    dict(B=2, K=3, V=4099, dtype="bf16", T=1.3, top_p=0.95, k=5),      # unaligned bf16 rows
+    dict(B=4, K=5, V=8200, dtype="bf16", T=0.6, top_p=0.8, k=64),      # aligned, ragged sketch tail
+    dict(B=2, K=16, V=20000, dtype="f32", T=1.0, top_p=1.0, k=256),    # top_p = 1, largest payload
+    dict(B=5, K=1, V=65544, dtype="bf16", T=2.0, top_p=0.99, k=16),    # flat rows: exact fallback
+    dict(B=2, K=4, V=2, dtype="f32", T=1.0, top_p=0.5, k=2),           # smallest vocabulary
+    dict(B=3, K=3, V=50000, dtype="bf16", T=0.3, top_p=0.05, k=8, rho=0.95),  # one-id nucleus
+    dict(B=2, K=2, V=300000, dtype="bf16", T=0.9, top_p=0.9, k=32, zipf=True),  # larger sketch groups
+]
+
+
+@pytest.mark.parametrize("cfg", RAGGED, ids=lambda c: f"{c['dtype']}_V{c['V']}_p{c['top_p']}")
+def test_ragged_sizes(A, orc, cfg):
+    cfg = dict(cfg)
+    w = gen.make_workload(cfg.pop("B"), cfg.pop("K"), cfg.pop("V"), seed=11, **cfg)
+    inp = gen.generate(w)
+    g, o, res = check_all(A, orc, inp, w)
+    F = tuple(min(3, w.V - 1) for _ in range(w.K))
+    check_cache(A, orc, inp, F, g)
+
+
+def test_sparsify_matches_oracle(A, orc):
+    w = gen.make_workload(6, 3, 33000, "bf16", T=0.8, top_p=0.9, k=40, seed=3)
+    inp = gen.generate(w)
+    z = torch.from_numpy(inp["z"].view(np.int16)).cuda().view(torch.bfloat16)
+    out = _np(A.sparsify(z, w.T, w.top_p, w.k))
+    torch.cuda.synchronize()
+    o = orc.sparsify(inp["z"], w.T, w.top_p, w.k)
+    o["topk_ids"] = o["topk_ids"].reshape(out["topk_ids"].shape)
+    parity.compare_payload(out, o, w.top_p, True)
+    np.testing.assert_array_equal(out["row_status"].reshape(-1), o["row_status"])
+
+
+def test_unaligned_pointer_takes_general_path(A, orc):
+    w = gen.make_workload(2, 3, 8192, "f32", T=0.9, top_p=0.9, k=20, seed=4)
+    inp = gen.generate(w)
+    z = torch.from_numpy(inp["z"]).cuda()
+    big = torch.empty(z.numel() + 1, dtype=torch.float32, device="cuda")
+    big[1:].copy_(z.reshape(-1))
+    zu = big[1:].view(z.shape)                       # 4-byte aligned, not 16
+    q, xt, u = (torch.from_numpy(inp[key]).cuda() for key in ("q", "xt", "u"))
+    g = _np(A.verify(zu, q, xt, u, w.T, w.top_p, w.k))
+    o = orc.verify(inp["z"], inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
+    parity.compare_verify(inp, g, o, w.top_p, False, w.k)
+
+
+def test_deterministic_rerun(A):
+    w = gen.WORKLOADS["b16_k8_v32000_f32"]
+    inp = gen.generate(w)
+    a = run_gpu(A, inp, w, w.k)
+    b = run_gpu(A, inp, w, w.k)
+    for key in a:
+        np.testing.assert_array_equal(a[key], b[key])
+
+
+# ---------------------------------------------------------------------------
+# degenerate inputs
+
+
+def _edge_inputs():
+    w = gen.make_workload(8, 3, 4096, "f32", T=1.0, top_p=0.9, k=8, seed=21)
+    return w, gen.generate(w)
+
+
+def test_nonfinite_rows_and_bad_drafts(A, orc):
+    w, inp = _edge_inputs()
+    z, q, xt, u = (inp[key].copy() for key in ("z", "q", "xt", "u"))
+    z[0, 1, 17] = np.nan                 # NaN logit in row 1 of seq 0
+    z[1, 0, :] = -np.inf                 # a row with no finite logit
+    z[2, 2, 5] = np.inf                  # +inf logit
+    z[3, 0, ::2] = -np.inf               # half masked: allowed
+    xt[4, 0] = 4096 + 3                  # out-of-range draft token
+    q[5, 0, xt[5, 0]] = 0.0              # drafted an id with zero draft probability
+    q[6, 1, 100] = np.nan                # NaN in a draft row (hits the residual if pi = 1)
+    u[6, 0] = 1e-7                       # make position 0 accept for seq 6
+    z[7, :, :] = 0.5                     # constant rows: ties everywhere
+    inp2 = dict(z=z, q=q, xt=xt, u=u)
+    g = run_gpu(A, inp2, w, w.k)
+    o = orc.verify(z, q, xt, u, w.T, w.top_p, w.k)
+    res = parity.compare_verify(inp2, g, o, w.top_p, False, w.k)
+    assert g["row_status"][0, 1] & 1 and g["row_status"][1, 0] & 1 and g["row_status"][2, 2] & 1
+    assert g["row_status"][4, 0] & 2 and g["row_status"][5, 0] & 2
+    assert res["checked_seqs"] >= 6
+
+
+def test_top_p_boundary_cases(A, orc):
+    w, inp = _edge_inputs()
+    for top_p in (1e-6, 0.5, 0.999999, 1.0):
+        w2 = gen.make_workload(w.B, w.K, w.V, "f32", T=1.0, top_p=top_p, k=8, seed=21)
+        g = run_gpu(A, inp, w2, 8)
+        o = orc.verify(inp["z"], inp["q"], inp["xt"], inp["u"], 1.0, top_p, 8)
+        parity.compare_verify(inp, g, o, top_p, False, 8)
+
+
+def test_cache_fanout_above_one_pass(A, orc):
+    w = gen.make_workload(3, 4, 5000, "f32", T=1.2, top_p=1.0, k=4, seed=31)
+    inp = gen.generate(w)
+    for F in ((20, 0, 9, 1), (64, 64, 64, 64), (0, 0, 0, 1)):
+        check_cache(A, orc, inp, F)
+    q = inp["q"].copy()
+    q[0, 0, inp["xt"][0, 0]] = 1.0       # 1 - q(x~) = 0: all branches padded
+    inp2 = dict(inp, q=q)
+    bt = check_cache(A, orc, inp2, (5, 5, 5, 5))
+    assert (bt[0, :5] == -1).all()
+
+
+def test_invalid_arguments_are_rejected(A):
+    z = torch.zeros(1, 3, 16, device="cuda")
+    q = torch.full((1, 2, 16), 1 / 16, device="cuda")
+    xt = torch.zeros(1, 2, dtype=torch.int32, device="cuda")
+    u = torch.full((1, 3), 0.5, device="cuda")
+    with pytest.raises(A.AcespecError) as e:
+        A.verify(z, q, xt, u, 0.0, 0.9, 4)
+    assert e.value.code == 2                 # T = 0 (greedy) unsupported
+    for T, tp, k in ((-1.0, 0.9, 4), (1.0, 0.0, 4), (1.0, 1.5, 4), (1.0, 0.9, 17), (float("nan"), 0.9, 4)):
+        with pytest.raises(A.AcespecError) as e:
+            A.verify(z, q, xt, u, T, tp, k)
+        assert e.value.code == 1
