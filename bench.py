@@ -1,0 +1,467 @@
+#!/usr/bin/env python
+"""Benchmark of the AceSpec hot path on GB300.
+
+One step = one pass of the whole path over one batch: aces_verify (temperature
+softmax, nucleus, accept tests, first rejection, residual/bonus draw, fused
+sparse top-k payload) + aces_cache_build (per-depth branch cache) +
+aces_cache_lookup, on the B=256, K=16, V=256000 bfloat16 workload
+(T=0.6, top_p=0.8, k=128, F=[4]*16).  Inputs (6.4 GB) are larger than L2, so
+no flush is needed between steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl acespec|reference]
+
+Prints one JSON line on rank 0.  With N > 1 (torchrun) every rank processes
+its own B sequences (weak scaling, no collective on the data path) and the
+timing is the max over ranks.  `--impl reference` times the float64 CPU
+oracle on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import glob
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verified rows/s and achieved HBM GB/s (fraction of GB300 peak) for verify+sparsify"
+WORKLOAD = "b256_k16_v256000_bf16"
+SWEEP_B = (32, 64, 128, 256)
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region: NVML polled at ~1 ms plus nvidia-smi (read only)
+class ClockSampler:
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, pci_bus_id: str | None):
+        self.samples = []
+        self.smi_lines = []
+        self._stop = threading.Event()
+        self._nvml = None
+        self._h = None
+        self.max_mhz = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() == 0:
+                h = ctypes.c_void_p()
+                ok = -1
+                if pci_bus_id:
+                    ok = nv.nvmlDeviceGetHandleByPciBusId_v2(pci_bus_id.encode(), ctypes.byref(h))
+                if ok != 0:
+                    ok = nv.nvmlDeviceGetHandleByIndex_v2(0, ctypes.byref(h))
+                if ok == 0:
+                    self._nvml, self._h = nv, h
+                    mx = ctypes.c_uint()
+                    if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+                        self.max_mhz = mx.value
+        except OSError:
+            pass
+        self._smi = None
+
+    def _poll(self):
+        nv, h = self._nvml, self._h
+        clk = ctypes.c_uint()
+        rs = ctypes.c_ulonglong()
+        pw = ctypes.c_uint()
+        while not self._stop.is_set():
+            if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0:
+                r = rs.value if nv.nvmlDeviceGetCurrentClocksEventReasons(h, ctypes.byref(rs)) == 0 else 0
+                p = pw.value / 1000.0 if nv.nvmlDeviceGetPowerUsage(h, ctypes.byref(pw)) == 0 else None
+                self.samples.append((clk.value, r, p))
+            time.sleep(0.001)
+
+    def __enter__(self):
+        try:
+            q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+            self._smi = subprocess.Popen(["nvidia-smi", f"--query-gpu={q}", "--format=csv,noheader",
+                                          "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                         text=True)
+        except OSError:
+            self._smi = None
+        if self._nvml is not None:
+            self._t = threading.Thread(target=self._poll, daemon=True)
+            self._t.start()
+        return self
+
+    def __exit__(self, *exc):
+        self._stop.set()
+        if self._nvml is not None:
+            self._t.join()
+        if self._smi is not None:
+            self._smi.terminate()
+            try:
+                out, _ = self._smi.communicate(timeout=5)
+                self.smi_lines = [ln for ln in out.splitlines() if ln.strip()]
+            except subprocess.TimeoutExpired:
+                self._smi.kill()
+        return False
+
+    def summary(self):
+        mhz = [s[0] for s in self.samples]
+        reasons = set()
+        for _, r, _ in self.samples:
+            for bit, name in self.REASONS.items():
+                if r & bit:
+                    reasons.add(name)
+        smi_mhz = []
+        for ln in self.smi_lines:
+            f = [x.strip() for x in ln.split(",")]
+            try:
+                smi_mhz.append(float(f[1].split()[0]))
+                if self.max_mhz is None:
+                    self.max_mhz = float(f[2].split()[0])
+                for name, col in (("hw_slowdown", 5), ("hw_thermal_slowdown", 6), ("sw_thermal_slowdown", 7),
+                                  ("sw_power_cap", 8)):
+                    if f[col].lower() == "active":
+                        reasons.add(name)
+            except (IndexError, ValueError):
+                pass
+        allm = mhz or smi_mhz
+        pw = [s[2] for s in self.samples if s[2] is not None]
+        return {"sm_mhz": statistics.median(allm) if allm else None, "sm_max_mhz": self.max_mhz,
+                "reasons": sorted(reasons), "samples": len(mhz), "smi_samples": len(smi_mhz),
+                "power_w_max": max(pw) if pw else None}
+
+
+# ---------------------------------------------------------------------------
+def measured_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2609_02514_gb300", "csrc", "*"))):
+        h.update(open(f, "rb").read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel: str, units: float):
+    """DRAM bytes per launch from the committed ncu summary, scaled to the
+    timed launch's units; None when the kernels changed since the capture."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        d = json.load(open(p))
+    except (OSError, ValueError):
+        return None
+    if d.get("source_hash") != kernel_source_hash():
+        return None
+    e = d.get("kernels", {}).get(kernel)
+    if not e:
+        return None
+    return e["dram_bytes"] * units / e["units"]
+
+
+def verify_bytes(B, K, V, k, zsize, n_rej):
+    """Algorithmic bytes of one aces_verify call with a payload of k."""
+    rd = B * (K + 1) * V * zsize + n_rej * V * 4 + B * K * 12 + B * 4
+    wr = B * (K + 1) * (8 * k + 4) + B * 8 + B * (K + 1) * 4
+    return rd + wr
+
+
+def cache_bytes(B, K, V, S):
+    return B * K * V * 4 + B * K * 4 + B * S * 8
+
+
+# ---------------------------------------------------------------------------
+def init_dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def reference_arm(args, ws, rank):
+    """Times the float64 CPU oracle as it stands on a bounded sample."""
+    if rank != 0:
+        return
+    import numpy as np  # noqa: F401
+
+    import gen
+    from oracle import oracle as O
+    O.build()
+    w = gen.WORKLOADS[args.workload]
+    cores = O.num_threads()
+    nseq = max(1, min(cores, w.B, args.ref_seqs))
+    inp = gen.generate_sequences(w, range(nseq), workers=min(16, os.cpu_count() or 1))
+    rows = nseq * (w.K + 1)
+
+    def step():
+        O.verify(inp["z"], inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
+        O.cache_build(inp["q"], inp["xt"], w.F)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    val = rows * args.steps / dt
+    sample = f"{nseq} of {w.B} sequences ({rows} target rows + {nseq * w.K} draft rows) per step"
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": val, "unit": "rows/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_of(w),
+        "cpu_baseline": {"value": val, "unit": "rows/s", "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": val, "unit": "rows/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def config_of(w):
+    return {"workload": w.name if w.B == gen_B(w) else f"{w.name} (first {w.B} sequences)", "B": w.B, "K": w.K, "V": w.V, "logits": w.dtype, "T": w.T, "top_p": w.top_p,
+            "k": w.k, "F": list(w.F), "l2": "inputs (z 2.2 GB + q 4.2 GB) exceed the 129 MB L2; no flush",
+            "parallelism": "one process per GPU, sequences sharded, no collective"}
+
+
+def gen_B(w):
+    import gen
+    return gen.WORKLOADS[w.name].B
+
+
+def cpu_baseline(w, inp):
+    from oracle import oracle as O
+    O.build()
+    cores = O.num_threads()
+    nseq = min(w.B, max(1, cores))
+    sub = {k: inp[k][:nseq] for k in ("z", "q", "xt", "u")}
+    t0 = time.perf_counter()
+    O.verify(sub["z"], sub["q"], sub["xt"], sub["u"], w.T, w.top_p, w.k)
+    O.cache_build(sub["q"], sub["xt"], w.F)
+    dt = time.perf_counter() - t0
+    rows = nseq * (w.K + 1)
+    return {"value": rows / dt, "unit": "rows/s", "cores": cores, "kind": "oracle",
+            "sample": f"{nseq} of {w.B} sequences: verify+sparsify ({rows} rows) and cache build "
+                      f"({nseq * w.K} rows), OpenMP over sequences, {dt:.1f} s"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="acespec", choices=["acespec", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--ref-seqs", type=int, default=16)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=0)
+    ap.add_argument("--B", type=int, default=0, help="use only the first B sequences (small profiling runs)")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    ws, rank, local = init_dist()
+
+    if args.impl == "reference":
+        reference_arm(args, ws, rank)
+        return
+
+    import numpy as np
+    import torch
+
+    import gen
+    import paper_2609_02514_gb300 as A
+
+    w = gen.WORKLOADS[args.workload]
+    if args.B:
+        import dataclasses
+        w = dataclasses.replace(w, B=min(args.B, w.B))
+    # host inputs first (spawn pool), this rank's shard of sequences
+    inp = gen.generate_sequences(w, range(rank * w.B, (rank + 1) * w.B), workers=min(16, os.cpu_count() or 1))
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+    A.load()
+    B, K, V, k = w.B, w.K, w.V, w.k
+    S = int(sum(w.F))
+    zsize = 2 if w.dtype == "bf16" else 4
+
+    # pinned host copies (e2e) and device-resident inputs
+    zh = torch.from_numpy(inp["z"].view(np.int16)).view(torch.bfloat16) if w.dtype == "bf16" \
+        else torch.from_numpy(inp["z"])
+    host = {"z": zh.pin_memory(), "q": torch.from_numpy(inp["q"]).pin_memory(),
+            "xt": torch.from_numpy(inp["xt"]).pin_memory(), "u": torch.from_numpy(inp["u"]).pin_memory()}
+    d = {key: t.to(dev) for key, t in host.items()}
+    out = A.verify(d["z"], d["q"], d["xt"], d["u"], w.T, w.top_p, k)
+    cache = A.cache_build(d["q"], d["xt"], w.F)
+    slot = A.cache_lookup(cache["branch_tok"], w.F, out["accept_len"], out["out_token"])
+    wsb = torch.empty(A.workspace_bytes(B, K, V, k), dtype=torch.uint8, device=dev)
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        A.verify(d["z"], d["q"], d["xt"], d["u"], w.T, w.top_p, k, out=out, workspace=wsb)
+        if ev is not None:
+            ev[1].record(stream)
+        A.cache_build(d["q"], d["xt"], w.F, out=cache)
+        if ev is not None:
+            ev[2].record(stream)
+        A.cache_lookup(cache["branch_tok"], w.F, out["accept_len"], out["out_token"], out=slot)
+        if ev is not None:
+            ev[3].record(stream)
+
+    def barrier():
+        if pg is not None:
+            pg.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(x):
+        if pg is None:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        return float(t.item())
+
+    for _ in range(args.warmup):
+        step()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    pci = None
+    try:
+        pci = torch.cuda.get_device_properties(dev).pci_bus_id  # may not exist on every torch
+    except AttributeError:
+        pass
+    barrier()
+    with ClockSampler(pci) as clocks:
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for i in range(args.steps):
+            step(evs[i])
+        t1.record(stream)
+        barrier()
+    ms_total = max_over_ranks(t0.elapsed_time(t1))
+    ms_step = ms_total / args.steps
+    part_ms = {
+        "verify_sparsify": statistics.mean(e[0].elapsed_time(e[1]) for e in evs),
+        "cache_build": statistics.mean(e[1].elapsed_time(e[2]) for e in evs),
+        "cache_lookup": statistics.mean(e[2].elapsed_time(e[3]) for e in evs),
+    }
+    rows = B * (K + 1)
+    value = ws * rows / (ms_step * 1e-3)
+
+    al = out["accept_len"].cpu().numpy()
+    n_rej = int((al < K).sum())
+    fb = int(wsb[:4].view(torch.int32).item())
+    peak, peak_kind = measured_peak()
+    vb = verify_bytes(B, K, V, k, zsize, n_rej)
+    cb = cache_bytes(B, K, V, S)
+    parts = {
+        "verify_sparsify": {"ms": part_ms["verify_sparsify"], "rows_per_s": rows / (part_ms["verify_sparsify"] * 1e-3),
+                            "alg_bytes": vb, "gbs": vb / (part_ms["verify_sparsify"] * 1e-3) / 1e9,
+                            "kernels": ["k_rows_fast", "k_rows_general", "k_resolve"],
+                            "rows_on_general_path": fb, "rejecting_sequences": n_rej},
+        "cache_build": {"ms": part_ms["cache_build"], "alg_bytes": cb,
+                        "gbs": cb / (part_ms["cache_build"] * 1e-3) / 1e9, "kernels": ["k_cache_build"]},
+        "cache_lookup": {"ms": part_ms["cache_lookup"], "kernels": ["k_cache_lookup"]},
+    }
+    for p in parts.values():
+        if "gbs" in p:
+            p["frac_of_peak"] = p["gbs"] / peak
+    dom = max(("verify_sparsify", "cache_build"), key=lambda n: part_ms[n])
+    dom_kernel = "aces_verify" if dom == "verify_sparsify" else "k_cache_build"
+    roof = {"bound": "hbm", "kernel": dom_kernel, "achieved": parts[dom]["gbs"], "peak": peak, "unit": "GB/s",
+            "frac": parts[dom]["gbs"] / peak, "peak_kind": peak_kind,
+            "traffic": profiled_traffic(dom_kernel, B)}
+    roof_v = {"bound": "hbm", "kernel": "aces_verify", "achieved": parts["verify_sparsify"]["gbs"], "peak": peak,
+              "unit": "GB/s", "frac": parts["verify_sparsify"]["gbs"] / peak, "peak_kind": peak_kind,
+              "traffic": profiled_traffic("aces_verify", B)}
+
+    # B sweep at V = 256000 (verify + sparsify only, device-resident inputs)
+    sweep = []
+    if not args.no_sweep and rank == 0:
+        for bs in SWEEP_B:
+            if bs > B:
+                continue
+            sub = {key: d[key][:bs] for key in ("z", "q", "xt", "u")}
+            o2 = A.verify(sub["z"], sub["q"], sub["xt"], sub["u"], w.T, w.top_p, k)
+            ws2 = torch.empty(A.workspace_bytes(bs, K, V, k), dtype=torch.uint8, device=dev)
+            for _ in range(3):
+                A.verify(sub["z"], sub["q"], sub["xt"], sub["u"], w.T, w.top_p, k, out=o2, workspace=ws2)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            n = 10
+            e0.record(stream)
+            for _ in range(n):
+                A.verify(sub["z"], sub["q"], sub["xt"], sub["u"], w.T, w.top_p, k, out=o2, workspace=ws2)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1) / n
+            nr = int((o2["accept_len"] < K).sum().item())
+            by = verify_bytes(bs, K, V, k, zsize, nr)
+            sweep.append({"B": bs, "ms": ms, "rows_per_s": bs * (K + 1) / (ms * 1e-3), "gbs": by / (ms * 1e-3) / 1e9,
+                          "frac_of_peak": by / (ms * 1e-3) / 1e9 / peak})
+
+    # end to end through the public API: pinned host inputs in, results out
+    e2e_steps = args.e2e_steps or args.steps
+    res_keys = ["accept_len", "out_token", "row_status", "topk_ids", "topk_probs", "tail_mass"]
+    host_out = {key: torch.empty_like(out[key], device="cpu").pin_memory() for key in res_keys}
+    host_cache = {key: torch.empty_like(cache[key], device="cpu").pin_memory() for key in cache}
+    host_slot = torch.empty_like(slot, device="cpu").pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = sum(t.numel() * t.element_size() for t in host_out.values()) + \
+        sum(t.numel() * t.element_size() for t in host_cache.values()) + host_slot.numel() * 4
+
+    def e2e_step():
+        for key in host:
+            d[key].copy_(host[key], non_blocking=True)
+        step()
+        for key in res_keys:
+            host_out[key].copy_(out[key], non_blocking=True)
+        for key in cache:
+            host_cache[key].copy_(cache[key], non_blocking=True)
+        host_slot.copy_(slot, non_blocking=True)
+        stream.synchronize()
+
+    for _ in range(2):
+        e2e_step()
+    barrier()
+    t = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    barrier()
+    e2e_s = max_over_ranks((time.perf_counter() - t) / e2e_steps)
+    e2e = {"value": ws * rows / e2e_s, "unit": "rows/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+           "ms_per_step": e2e_s * 1e3}
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, inp)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": config_of(w),
+            "roofline": roof, "roofline_verify_sparsify": roof_v, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": 5 * args.steps, "clocks": clocks.summary(), "parts": parts, "sweep": sweep,
+        }
+        print(json.dumps(line), flush=True)
+    if pg is not None:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

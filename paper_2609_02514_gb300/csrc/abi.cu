@@ -45,21 +45,19 @@ aces_status run_rows(RowArgs &a, aces_dtype dt, cudaStream_t s) {
     const bool vec = aligned16(a.logits) && ((size_t)a.V * es) % 16 == 0;
     const int nsm = sm_count();
     if (cudaMemsetAsync(a.ws.fb_count, 0, 16, s) != cudaSuccess) return ACES_ERR_CUDA;
-    if (vec) {
-        const int epc = dt == ACES_BF16 ? 8 : 4;
-        const int nch = a.V / epc;
-        const int gmax = dt == ACES_BF16 ? 8 : 16;
-        int gc = 2;
-        while (gc < gmax && (nch + gc - 1) / gc > SKETCH_CAP) gc *= 2;
-        a.ng = (nch + gc - 1) / gc;
-        const size_t smem = align16((size_t)a.ng * 4) + (size_t)CAND_CAP * 8;
-        if (launch_rows_fast(a, dt, gc, smem, s) != cudaSuccess) return ACES_ERR_CUDA;
+    const int gc = vec ? rows_fast_gc(dt, a.V) : 0;
+    if (gc > 0) {
+        const int nch = (int)((size_t)a.V * es / 16);
+        a.ng = (nch + gc - 1) / gc;  // sketch groups of gc 16-byte chunks
+        const size_t smem = rows_fast_smem(dt, gc, nch);
+        const int pgrid = a.rows < 2 * nsm ? a.rows : 2 * nsm;  // persistent: rows claimed dynamically
+        if (launch_rows_fast(a, dt, gc, smem, pgrid, s) != cudaSuccess) return ACES_ERR_CUDA;
         int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
         if (launch_rows_general(a, dt, true, 0, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
     } else {
         a.ng = 0;
         int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
-        if (launch_rows_general(a, dt, false, 1, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
+        if (launch_rows_general(a, dt, vec, 1, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
     }
     return ACES_OK;
 }
@@ -73,7 +71,7 @@ size_t aces_workspace_bytes(int B, int K, int V, int k) {
         return 0;
     long long rows = (long long)B * (K + 1);
     if (rows > INT_MAX / 2) return 0;
-    return ws_bytes((int)rows, B * K);
+    return ws_bytes((int)rows, B, K);
 }
 
 aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *draft_probs,
@@ -109,7 +107,7 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
     a.topk_probs = topk_probs;
     a.tail = tail_mass;
     a.row_status = row_status;
-    a.ws = ws_carve(workspace, rows, B * K);
+    a.ws = ws_carve(workspace, rows, B, K);
     a.ng = 0;
     st = run_rows(a, dt, s);
     if (st != ACES_OK) return st;
@@ -156,7 +154,7 @@ aces_status aces_sparsify(const void *target_logits, aces_dtype dt, int rows, in
     a.topk_probs = topk_probs;
     a.tail = tail_mass;
     a.row_status = row_status;
-    a.ws = ws_carve(workspace, rows, 0);
+    a.ws = ws_carve(workspace, rows, rows, 0);
     a.ng = 0;
     return run_rows(a, dt, reinterpret_cast<cudaStream_t>(stream));
 }

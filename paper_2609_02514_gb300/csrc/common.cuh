@@ -11,7 +11,6 @@ namespace aces {
 constexpr int NT = 512;             // threads per CTA for every row kernel
 constexpr int NWARP = NT / 32;
 constexpr int SKETCH_CAP = 16384;   // max sketch groups per row (fast path)
-constexpr int CAND_CAP = 4096;      // max candidates per row (fast path)
 constexpr int NBIN = 256;           // sketch bins of width T/8 below the max
 constexpr int BIN_PER_T = 8;
 
@@ -21,9 +20,9 @@ constexpr int RS_NONFINITE = 2;
 
 // Per-row state written by the row kernels and read by the resolve kernel.
 struct RowStat {
-    float m;                 // row max logit
+    float kref;              // log2 reference: masses are 2^(z*c - kref)
     float c;                 // log2(e) / T
-    double S_nuc;            // nucleus mass, in units of exp((z - m)/T)
+    double S_nuc;            // nucleus mass in the same units
     unsigned long long cut;  // order value of the last nucleus id
     int flags;
     int pad;
@@ -114,17 +113,21 @@ __device__ __forceinline__ unsigned long long warp_max(unsigned long long v) {
     return v;
 }
 
-// `red` must hold NWARP entries; every thread gets the result.
-template <class T, class Op>
-__device__ __forceinline__ T block_reduce(T v, T *red, Op op) {
+// `red` must hold NTH/32 entries; every thread gets the result.
+template <int NTH, class T, class Op>
+__device__ __forceinline__ T block_reduce_n(T v, T *red, Op op) {
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     v = op(v);
     __syncthreads();
     if (lane == 0) red[wid] = v;
     __syncthreads();
     T r = red[0];
-    for (int i = 1; i < NWARP; ++i) r = op.combine(r, red[i]);
+    for (int i = 1; i < NTH / 32; ++i) r = op.combine(r, red[i]);
     return r;
+}
+template <class T, class Op>
+__device__ __forceinline__ T block_reduce(T v, T *red, Op op) {
+    return block_reduce_n<NT>(v, red, op);
 }
 struct SumD {
     __device__ double operator()(double v) const { return warp_sum(v); }
@@ -145,11 +148,12 @@ struct MaxU64 {
     }
 };
 
-// Exclusive scan over the block of one u64 per thread; `red` holds NWARP
+// Exclusive scan over the block of one u64 per thread; `red` holds NTH/32
 // entries.  Returns the exclusive prefix; *total gets the block sum.
-__device__ __forceinline__ unsigned long long block_exscan(unsigned long long v,
-                                                           unsigned long long *red,
-                                                           unsigned long long *total) {
+template <int NTH>
+__device__ __forceinline__ unsigned long long block_exscan_n(unsigned long long v,
+                                                             unsigned long long *red,
+                                                             unsigned long long *total) {
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     unsigned long long inc = v;
     for (int o = 1; o < 32; o <<= 1) {
@@ -160,7 +164,7 @@ __device__ __forceinline__ unsigned long long block_exscan(unsigned long long v,
     if (lane == 31) red[wid] = inc;
     __syncthreads();
     unsigned long long base = 0, all = 0;
-    for (int i = 0; i < NWARP; ++i) {
+    for (int i = 0; i < NTH / 32; ++i) {
         if (i < wid) base += red[i];
         all += red[i];
     }
@@ -212,11 +216,74 @@ __host__ __device__ __forceinline__ int next_pow2(int n) {
     return p;
 }
 
-// fixed point for exact, order-independent sums of probabilities in [0, 1]
+// fixed point for exact, order-independent sums of probabilities: floor(x * 2^40)
+// for 0 <= x < 2^23, from the float's bits with integer operations only
 constexpr float FX_SCALE = 1099511627776.0f;  // 2^40
 __device__ __forceinline__ unsigned long long to_fx(float x) {
-    return __float2ull_rn(x * FX_SCALE);
+    const uint32_t u = __float_as_uint(x);
+    const uint32_t be = u >> 23;                      // biased exponent (sign is 0)
+    if (be == 0u) return 0ull;
+    const unsigned long long mant = (unsigned long long)((u & 0x7FFFFFu) | 0x800000u);
+    const int sh = (int)be - 110;                     // x * 2^40 = mant * 2^(be - 127 - 23 + 40)
+    return sh >= 0 ? (mant << sh) : (sh > -64 ? (mant >> (-sh)) : 0ull);
 }
+
+// ---------------------------------------------------------------------------
+// mbarrier and bulk async copy (global -> shared), CTA scope
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(unsigned long long *bar, unsigned count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(unsigned long long *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(unsigned long long *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(unsigned long long *bar, uint32_t phase) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_u32(bar)), "r"(phase)
+        : "memory");
+    return done != 0u;
+}
+// Waits for the phase with the given parity to complete; gives up after
+// about one second (2^31 SM clock cycles) and returns false.
+__device__ __forceinline__ bool mbar_wait_bounded(unsigned long long *bar, uint32_t phase) {
+    if (mbar_try_wait(bar, phase)) return true;
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, phase)) {
+        if (clock64() - t0 > (1ll << 31)) return false;
+    }
+    return true;
+}
+// bytes and both addresses must be multiples of 16
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, unsigned long long *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Exact sums of one vocabulary segment of a sequence's row pi (2^-40 units).
+struct SegSum {
+    unsigned long long r;  // residual max(0, p - q)
+    unsigned long long p;  // p itself
+    int bad;               // a NaN / negative draft probability was seen
+    int pad;
+};
+constexpr int NSEG_MAX = 16;
 
 // Workspace layout (all offsets 16-byte aligned)
 struct Workspace {
@@ -224,13 +291,15 @@ struct Workspace {
     RowStat *stats;   // [rows]
     int *acc;         // [B*K] accept bits
     int *fb_list;     // [rows]
+    SegSum *seg;      // [B*NSEG_MAX] (verify only)
 };
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
-__host__ __device__ inline size_t ws_bytes(int rows, int nacc) {
-    return 16 + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nacc * 4) +
-           align16((size_t)rows * 4);
+// rows = B*(K+1) target rows; nseq = B sequences with K draft positions (0 for sparsify)
+__host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K) {
+    return 16 + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
+           align16((size_t)rows * 4) + (K > 0 ? align16((size_t)nseq * NSEG_MAX * sizeof(SegSum)) : 0);
 }
-__host__ __device__ inline Workspace ws_carve(void *base, int rows, int nacc) {
+__host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K) {
     char *p = (char *)base;
     Workspace w;
     w.fb_count = (int *)p;
@@ -238,8 +307,10 @@ __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nacc) {
     w.stats = (RowStat *)p;
     p += align16((size_t)rows * sizeof(RowStat));
     w.acc = (int *)p;
-    p += align16((size_t)nacc * 4);
+    p += align16((size_t)nseq * K * 4);
     w.fb_list = (int *)p;
+    p += align16((size_t)rows * 4);
+    w.seg = K > 0 ? (SegSum *)p : nullptr;
     return w;
 }
 
@@ -284,8 +355,44 @@ struct CacheArgs {
     float *bp;
 };
 
+// Outputs of a row whose logits are not a distribution.
+template <int NTH>
+__device__ void nonfinite_row(const RowArgs &a, int r) {
+    const int tid = threadIdx.x;
+    for (int j = tid; j < a.k; j += NTH) {
+        a.topk_ids[(size_t)r * a.k + j] = -1;
+        a.topk_probs[(size_t)r * a.k + j] = 0.0f;
+    }
+    if (tid == 0) {
+        if (a.k > 0) a.tail[r] = 1.0f;
+        a.row_status[r] = ACES_ROW_NONFINITE;
+        if (a.K > 0) {
+            const int b = r / (a.K + 1), i = r % (a.K + 1);
+            if (i < a.K) a.ws.acc[(size_t)b * a.K + i] = 0;
+        }
+        RowStat s;
+        s.kref = 0.f;
+        s.c = a.c;
+        s.S_nuc = 1.0;
+        s.cut = 0;
+        s.flags = RS_NONFINITE;
+        s.pad = 0;
+        a.ws.stats[r] = s;
+    }
+}
+
+// Outputs of a row whose kernel gave up on a wait (never expected).
+template <int NTH>
+__device__ void timeout_row(const RowArgs &a, int r) {
+    nonfinite_row<NTH>(a, r);
+    __syncthreads();
+    if (threadIdx.x == 0) a.row_status[r] = ACES_ROW_TIMEOUT;
+}
+
 // host launchers (defined next to their kernels)
-cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, cudaStream_t s);
+size_t rows_fast_smem(int dt, int gc, int nch);
+int rows_fast_gc(int dt, int V);
+cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, int grid, cudaStream_t s);
 cudaError_t launch_rows_general(const RowArgs &a, int dt, bool vec, int direct, int grid, cudaStream_t s);
 cudaError_t launch_resolve(const ResolveArgs &a, int dt, bool vec, cudaStream_t s);
 cudaError_t launch_cache_build(const CacheArgs &a, bool vec, cudaStream_t s);

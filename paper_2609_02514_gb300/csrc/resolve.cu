@@ -1,0 +1,279 @@
+// Sequence step of AceSpec verification (Sec. III-B, Algorithm 1): the first
+// rejection index pi of each drafted chain and the token emitted at pi,
+// drawn from norm(max(0, p_pi - q_pi)) when pi < K (from p_pi itself when
+// that is all zero) or from p_K when the whole chain was accepted.
+//
+// The draw is the smallest id j whose prefix sum over ids 0..j exceeds
+// u[b, K] times the total.  Every probability enters as an integer in units
+// of 2^-40, so all partial sums are exact and independent of the order in
+// which threads add them; the segment sums of pass one and the prefix scan
+// of pass two therefore agree bit for bit.
+//
+//   k_resolve_seg   (B x nseg CTAs) segment sums of the residual and of p
+//   k_resolve_pick  (B CTAs) locates the segment holding the draw and scans
+//                   it in 2048-id tiles until the crossing id is found
+#include "common.cuh"
+
+namespace aces {
+
+constexpr int NTR = 256;
+constexpr int EPT = 8;               // consecutive ids per thread
+constexpr int TILE = NTR * EPT;
+
+// r_fx (residual) and p_fx of ids [x0, x0 + EPT); *bad on a NaN / negative q.
+template <int DT, bool VEC>
+__device__ __forceinline__ void mass_fx(const char *zrow, const float *qrow, int V, int x0, const RowStat &rs,
+                                        float inv_S, unsigned long long rf[EPT], unsigned long long pf[EPT],
+                                        int *bad) {
+    using E = Elem<DT>;
+    float zv[EPT], qv[EPT];
+    if (VEC && x0 + EPT <= V) {
+        if (DT == ACES_BF16) {
+            const uint4 w = ldg16(zrow + (size_t)x0 * 2);
+#pragma unroll
+            for (int e = 0; e < EPT; ++e) zv[e] = E::get(w, e);
+        } else {
+            const uint4 w0 = ldg16(zrow + (size_t)x0 * 4), w1 = ldg16(zrow + (size_t)x0 * 4 + 16);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                zv[e] = Elem<ACES_F32>::get(w0, e);
+                zv[e + 4] = Elem<ACES_F32>::get(w1, e);
+            }
+        }
+        if (qrow) {
+            const uint4 w0 = ldg16(qrow + x0), w1 = ldg16(qrow + x0 + 4);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                qv[e] = Elem<ACES_F32>::get(w0, e);
+                qv[e + 4] = Elem<ACES_F32>::get(w1, e);
+            }
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < EPT; ++e) {
+            const int x = x0 + e;
+            zv[e] = x < V ? E::load1(zrow, x) : -INFINITY;
+            qv[e] = (qrow && x < V) ? __ldg(qrow + x) : 0.0f;
+        }
+    }
+#pragma unroll
+    for (int e = 0; e < EPT; ++e) {
+        const int x = x0 + e;
+        const float v = zv[e];
+        const bool in = x < V && ((rs.flags & RS_ALL_IN) ? (v > -INFINITY)
+                                                         : (order_val(fkey(v), (uint32_t)x) >= rs.cut));
+        const float p = in ? ex2(fmaf(v, rs.c, -rs.kref)) * inv_S : 0.0f;
+        float rr = p;
+        if (qrow && x < V) {
+            const float qx = qv[e];
+            if (!(qx >= 0.0f)) *bad = 1;
+            rr = fmaxf(p - qx, 0.0f);
+        }
+        pf[e] = x < V ? to_fx(p) : 0ull;
+        rf[e] = x < V ? to_fx(rr) : 0ull;
+    }
+}
+
+__device__ __forceinline__ int first_reject(const Workspace &ws, int b, int K) {
+    int pi = K;
+    for (int i = 0; i < K; ++i)
+        if (!ws.acc[(size_t)b * K + i]) {
+            pi = i;
+            break;
+        }
+    return pi;
+}
+
+template <int DT, bool VEC>
+__global__ void __launch_bounds__(NTR) k_resolve_seg(ResolveArgs a, int nseg, int seglen) {
+    using E = Elem<DT>;
+    __shared__ int s_pi;
+    __shared__ unsigned long long red[NTR / 32];
+    __shared__ int s_bad;
+    const int b = blockIdx.x / nseg, sg = blockIdx.x % nseg, tid = threadIdx.x;
+    if (tid == 0) {
+        const int pi = first_reject(a.ws, b, a.K);
+        s_pi = pi;
+        s_bad = 0;
+        if (sg == 0) a.accept_len[b] = pi;
+    }
+    __syncthreads();
+    const int pi = s_pi;
+    const int r = b * (a.K + 1) + pi;
+    const RowStat rs = a.ws.stats[r];
+    SegSum *out = a.ws.seg + (size_t)b * nseg + sg;
+    if (rs.flags & RS_NONFINITE) {
+        if (tid == 0) *out = SegSum{0ull, 0ull, 0, 0};
+        return;
+    }
+    const char *zrow = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
+    const float *qrow = pi < a.K ? a.q + ((size_t)b * a.K + pi) * a.V : nullptr;
+    const float inv_S = (float)(1.0 / rs.S_nuc);
+    const int x_lo = sg * seglen, x_hi = min(a.V, x_lo + seglen);
+    unsigned long long sr = 0ull, sp = 0ull;
+    int bad = 0;
+    for (int x0 = x_lo + tid * EPT; x0 < x_hi; x0 += TILE) {
+        unsigned long long rf[EPT], pf[EPT];
+        mass_fx<DT, VEC>(zrow, qrow, x_hi, x0, rs, inv_S, rf, pf, &bad);
+#pragma unroll
+        for (int e = 0; e < EPT; ++e) {
+            sr += rf[e];
+            sp += pf[e];
+        }
+    }
+    if (bad) s_bad = 1;
+    const unsigned long long tr = block_reduce_n<NTR>(sr, red, SumU64());
+    const unsigned long long tp = block_reduce_n<NTR>(sp, red, SumU64());
+    if (tid == 0) *out = SegSum{tr, tp, s_bad, 0};
+}
+
+template <int DT, bool VEC>
+__global__ void __launch_bounds__(NTR) k_resolve_pick(ResolveArgs a, int nseg, int seglen) {
+    using E = Elem<DT>;
+    __shared__ unsigned long long red[NTR / 32];
+    __shared__ int s_seg, s_tok, s_done;
+    __shared__ unsigned long long s_base, s_thr;
+    __shared__ int s_mode, s_pi;
+    const int b = blockIdx.x, tid = threadIdx.x;
+    if (tid == 0) {
+        s_pi = first_reject(a.ws, b, a.K);
+        s_tok = -1;
+        s_done = 0;
+        s_seg = -1;
+    }
+    __syncthreads();
+    const int pi = s_pi;
+    const int r = b * (a.K + 1) + pi;
+    const RowStat rs = a.ws.stats[r];
+    if (rs.flags & RS_NONFINITE) {
+        if (tid == 0) a.out_token[b] = -1;
+        return;
+    }
+    const SegSum *seg = a.ws.seg + (size_t)b * nseg;
+    if (tid == 0) {
+        unsigned long long R = 0ull, P = 0ull;
+        int bad = 0;
+        for (int s = 0; s < nseg; ++s) {
+            R += seg[s].r;
+            P += seg[s].p;
+            bad |= seg[s].bad;
+        }
+        int mode = 0;
+        if (bad) {
+            a.row_status[r] |= ACES_ROW_BAD_Q;
+            s_done = 1;
+        } else {
+            if (R == 0ull) {
+                mode = 1;  // p <= q everywhere: draw from p itself
+                R = P;
+            }
+            if (R == 0ull) {
+                s_done = 1;
+            } else {
+                // thr = floor(u * R) exactly: u = M / 2^sh with a 24-bit integer M
+                const float uu = a.u[(size_t)b * (a.K + 1) + a.K];
+                int ex;
+                const float fr = frexpf(uu, &ex);
+                const unsigned long long M = (unsigned long long)ldexpf(fr, 24);
+                const int sh = 24 - ex;
+                const unsigned long long lo = M * R, hi = __umul64hi(M, R);
+                unsigned long long thr;
+                if (!(uu > 0.0f) || sh >= 128) thr = 0ull;
+                else if (sh >= 64) thr = hi >> (sh - 64);
+                else if (sh == 0) thr = lo;
+                else thr = (lo >> sh) | (hi << (64 - sh));
+                if (thr >= R) thr = R - 1ull;
+                unsigned long long base = 0ull;
+                int sg = nseg - 1;
+                for (int s = 0; s < nseg; ++s) {
+                    const unsigned long long v = mode ? seg[s].p : seg[s].r;
+                    if (base + v > thr) {
+                        sg = s;
+                        break;
+                    }
+                    base += v;
+                }
+                s_seg = sg;
+                s_base = base;
+                s_thr = thr;
+            }
+        }
+        s_mode = mode;
+    }
+    __syncthreads();
+    if (s_done) {
+        if (tid == 0) a.out_token[b] = -1;
+        return;
+    }
+    const char *zrow = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
+    const float *qrow = pi < a.K ? a.q + ((size_t)b * a.K + pi) * a.V : nullptr;
+    const float inv_S = (float)(1.0 / rs.S_nuc);
+    const int mode = s_mode;
+    const unsigned long long thr = s_thr;
+    const int x_lo = s_seg * seglen, x_hi = min(a.V, x_lo + seglen);
+    unsigned long long base = s_base;
+    for (int t0 = x_lo; t0 < x_hi; t0 += TILE) {
+        const int x0 = t0 + tid * EPT;
+        unsigned long long rf[EPT], pf[EPT];
+        int bad = 0;
+        if (x0 < x_hi) {
+            mass_fx<DT, VEC>(zrow, qrow, x_hi, x0, rs, inv_S, rf, pf, &bad);
+        } else {
+#pragma unroll
+            for (int e = 0; e < EPT; ++e) rf[e] = pf[e] = 0ull;
+        }
+        unsigned long long loc = 0ull;
+#pragma unroll
+        for (int e = 0; e < EPT; ++e) loc += mode ? pf[e] : rf[e];
+        unsigned long long tot;
+        const unsigned long long exs = block_exscan_n<NTR>(loc, red, &tot);
+        unsigned long long cum = base + exs;
+        if (cum <= thr && thr < cum + loc) {
+#pragma unroll
+            for (int e = 0; e < EPT; ++e) {
+                cum += mode ? pf[e] : rf[e];
+                if (cum > thr) {
+                    s_tok = x0 + e;
+                    break;
+                }
+            }
+            s_done = 1;
+        }
+        __syncthreads();
+        if (s_done) break;
+        base += tot;
+    }
+    if (tid == 0) a.out_token[b] = s_tok;
+}
+
+int resolve_segments(int V) {
+    int nseg = (V + 32767) / 32768;
+    return nseg < 1 ? 1 : (nseg > NSEG_MAX ? NSEG_MAX : nseg);
+}
+
+cudaError_t launch_resolve(const ResolveArgs &a, int dt, bool vec, cudaStream_t s) {
+    const int nseg = resolve_segments(a.V);
+    int seglen = (a.V + nseg - 1) / nseg;
+    seglen = (seglen + EPT - 1) / EPT * EPT;
+    const int g1 = a.B * nseg;
+    if (dt == ACES_BF16) {
+        if (vec) {
+            k_resolve_seg<ACES_BF16, true><<<g1, NTR, 0, s>>>(a, nseg, seglen);
+            k_resolve_pick<ACES_BF16, true><<<a.B, NTR, 0, s>>>(a, nseg, seglen);
+        } else {
+            k_resolve_seg<ACES_BF16, false><<<g1, NTR, 0, s>>>(a, nseg, seglen);
+            k_resolve_pick<ACES_BF16, false><<<a.B, NTR, 0, s>>>(a, nseg, seglen);
+        }
+    } else {
+        if (vec) {
+            k_resolve_seg<ACES_F32, true><<<g1, NTR, 0, s>>>(a, nseg, seglen);
+            k_resolve_pick<ACES_F32, true><<<a.B, NTR, 0, s>>>(a, nseg, seglen);
+        } else {
+            k_resolve_seg<ACES_F32, false><<<g1, NTR, 0, s>>>(a, nseg, seglen);
+            k_resolve_pick<ACES_F32, false><<<a.B, NTR, 0, s>>>(a, nseg, seglen);
+        }
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace aces

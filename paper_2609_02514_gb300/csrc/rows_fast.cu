@@ -1,0 +1,540 @@
+// Fast row kernel of the AceSpec cloud step (Sec. III-B: accept test and
+// packaging of the target distribution; Sec. V-C: compact payload; the
+// acceptance rule is the modified rejection sampling of Sec. II-A).
+//
+// One CTA of 256 threads per target row r = b*(K+1)+i, four CTAs per SM, so
+// that the short per-row epilogue of one row overlaps the HBM stream of the
+// others.
+//
+//   pass 1   every logit is read once from HBM with 16-byte loads (four in
+//            flight per thread): an online exp-sum in log2 units against an
+//            integer reference k_t = ceil(max z * log2(e)/T) (one FFMA and
+//            one ex2 per logit, rescales are exact powers of two), and the
+//            max of every group of 8*GC consecutive logits into a sketch.
+//   certify  groups are binned by (m - gmax) / (T/8); one max per group is
+//            a lower bound of the mass above a bin edge, so the first bin
+//            whose bound reaches top_p * S proves that the nucleus lies
+//            above that edge (for top_p = 1: the first bin holding k groups
+//            proves the top k lie above it).  Rows the sketch cannot certify
+//            go to the exact general kernel.
+//   select   ids above the edge are re-read (their groups only), bucketed by
+//            bin and ordered inside each bin by the 64-bit (logit, id)
+//            order; the nucleus crossing is found with exact fixed-point
+//            prefix sums in one warp.
+//   finish   payload (first k of the nucleus), tail mass, accept test of the
+//            draft token at this position, per-row state for the resolve
+//            kernels.
+#include <climits>
+#include <cuda_bf16.h>
+
+#include "common.cuh"
+
+namespace aces {
+
+constexpr int NTF = 256;
+constexpr int NWF = NTF / 32;
+constexpr int CAND_CAP_F = 2048;
+constexpr int MASK_GROUPS = 64;     // per-thread groups tracked in the high-group mask
+constexpr int MASK_BINS = 64;       // groups below this bin are remembered per thread
+constexpr int BUCKET_MAX = 32;      // largest bin sorted by insertion
+
+template <int DT> struct Sketch;
+template <> struct Sketch<ACES_F32> {
+    using T = uint32_t;
+    __device__ __forceinline__ static T enc(uint32_t key) { return key; }
+    __device__ __forceinline__ static float dec(T s) { return fkey_inv(s); }
+};
+template <> struct Sketch<ACES_BF16> {
+    using T = uint16_t;  // a bf16 key has 16 zero low bits
+    __device__ __forceinline__ static T enc(uint32_t key) { return (T)(key >> 16); }
+    __device__ __forceinline__ static float dec(T s) { return fkey_inv((uint32_t)s << 16); }
+};
+
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+    s = a + b;
+    const float bb = s - a;
+    e = (a - (s - bb)) + (b - bb);
+}
+
+// 2^d for an integer-valued d <= 0, exactly
+__device__ __forceinline__ float pow2_int(float d) {
+    return d >= -126.0f ? __int_as_float((127 + __float2int_rn(d)) << 23) : 0.0f;
+}
+
+template <int DT, int GC>
+__device__ __forceinline__ float group_max(const uint4 (&w)[GC]) {
+    if (DT == ACES_BF16) {
+        __nv_bfloat162 mx = *reinterpret_cast<const __nv_bfloat162 *>(&w[0].x);
+#pragma unroll
+        for (int j = 0; j < GC; ++j) {
+            const uint32_t wd[4] = {w[j].x, w[j].y, w[j].z, w[j].w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) mx = __hmax2(mx, *reinterpret_cast<const __nv_bfloat162 *>(&wd[q]));
+        }
+        const uint32_t u = *reinterpret_cast<const uint32_t *>(&mx);
+        return fmaxf(__uint_as_float(u << 16), __uint_as_float(u & 0xFFFF0000u));
+    } else {
+        float gm = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < GC; ++j)
+            gm = fmaxf(gm, fmaxf(fmaxf(__uint_as_float(w[j].x), __uint_as_float(w[j].y)),
+                                 fmaxf(__uint_as_float(w[j].z), __uint_as_float(w[j].w))));
+        return gm;
+    }
+}
+
+// sum over the group of 2^(z*c - k)
+template <int DT, int GC>
+__device__ __forceinline__ float group_expsum(const uint4 (&w)[GC], float c, float nk) {
+    using E = Elem<DT>;
+    float gs = 0.f;
+#pragma unroll
+    for (int j = 0; j < GC; ++j) {
+        float cs[E::EPC];
+#pragma unroll
+        for (int e = 0; e < E::EPC; ++e) cs[e] = ex2(fmaf(E::get(w[j], e), c, nk));
+#pragma unroll
+        for (int wdt = 1; wdt < E::EPC; wdt <<= 1)
+#pragma unroll
+            for (int e = 0; e < E::EPC; e += 2 * wdt) cs[e] += cs[e + wdt];
+        gs += cs[0];
+    }
+    return gs;
+}
+
+__device__ __forceinline__ void fallback_row(const RowArgs &a, int r) {
+    const int pos = atomicAdd(a.ws.fb_count, 1);
+    a.ws.fb_list[pos] = r;
+}
+
+template <int DT, int GC>
+__global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
+    using E = Elem<DT>;
+    using SK = typename Sketch<DT>::T;
+    constexpr int EPC = E::EPC;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int ng = a.ng;
+    SK *sketch = reinterpret_cast<SK *>(smem);
+    const size_t sk_bytes = align16((size_t)ng * sizeof(SK)) > (size_t)CAND_CAP_F * 8
+                                ? align16((size_t)ng * sizeof(SK)) : (size_t)CAND_CAP_F * 8;
+    unsigned long long *sorted = reinterpret_cast<unsigned long long *>(smem);  // after collection
+    unsigned long long *cand = reinterpret_cast<unsigned long long *>(smem + sk_bytes);
+    unsigned char *cbin = smem + sk_bytes + (size_t)CAND_CAP_F * 8;
+
+    __shared__ uint32_t bins[NBIN];
+    __shared__ uint32_t bstart[NBIN], bfill[NBIN];
+    __shared__ float redf[NWF], redk[NWF], redh[NWF], redl[NWF];
+    __shared__ int s_ncand, s_bc, s_nstar, s_L, s_bigbin;
+    __shared__ double s_S;
+    __shared__ unsigned long long s_cut, s_Snuc_fx, s_cumL_fx;
+
+    const int r = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const char *row = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
+    const int nch = a.V / EPC;
+    const uint32_t NI = E::NEG_INF_WORD;
+
+    // the draft token of this position, fetched early by thread 0
+    int xb = -1, bq = 0, iq = 0;
+    if (a.K > 0) {
+        bq = r / (a.K + 1);
+        iq = r % (a.K + 1);
+        if (tid == 0 && iq < a.K) xb = a.xt[(size_t)bq * a.K + iq];
+    }
+
+    // ---- pass 1 ----
+    float k_t = -1e30f, m_t = -INFINITY, s_t = 0.f, e_t = 0.f;
+    constexpr int GPI = GC >= 4 ? 1 : 2;  // groups per iteration: four 16-byte loads in flight
+    for (int g0 = tid; g0 < ng; g0 += NTF * GPI) {
+        uint4 w[GPI][GC];
+#pragma unroll
+        for (int h = 0; h < GPI; ++h) {
+            const int g = g0 + h * NTF;
+#pragma unroll
+            for (int j = 0; j < GC; ++j) {
+                const int cc = g * GC + j;
+                w[h][j] = (g < ng && cc < nch) ? ldg16(row + (size_t)cc * 16) : make_uint4(NI, NI, NI, NI);
+            }
+        }
+#pragma unroll
+        for (int h = 0; h < GPI; ++h) {
+            const int g = g0 + h * NTF;
+            const float gm = group_max<DT, GC>(w[h]);
+            m_t = fmaxf(m_t, gm);
+            const float gk = gm * a.c;
+            if (gk > k_t) {
+                const float nk = ceilf(gk);
+                const float sc = pow2_int(k_t - nk);
+                s_t *= sc;
+                e_t *= sc;
+                k_t = nk;
+            }
+            const float gs = group_expsum<DT, GC>(w[h], a.c, -k_t);
+            const float t = s_t + gs;
+            if (fabsf(s_t) >= fabsf(gs)) e_t += (s_t - t) + gs;
+            else e_t += (gs - t) + s_t;
+            s_t = t;
+            if (g < ng) sketch[g] = Sketch<DT>::enc(fkey(gm));
+        }
+    }
+    // dependent loads of the accept test, consumed at the end
+    float zx = 0.f, qx = 0.f;
+    if (xb >= 0 && xb < a.V) {
+        zx = E::load1(row, xb);
+        qx = __ldg(a.q + ((size_t)bq * a.K + iq) * a.V + xb);
+    }
+
+    // ---- row max, reference and exp-sum (fp32 two-sum tree, fp64 in thread 0) ----
+    {
+        const float mw = warp_max(m_t), kw = warp_max(k_t);
+        if (lane == 0) {
+            redf[wid] = mw;
+            redk[wid] = kw;
+        }
+    }
+    for (int i = tid; i < NBIN; i += NTF) bins[i] = 0u;
+    __syncthreads();
+    float m = redf[0], kref = redk[0];
+#pragma unroll
+    for (int i = 1; i < NWF; ++i) {
+        m = fmaxf(m, redf[i]);
+        kref = fmaxf(kref, redk[i]);
+    }
+    {
+        const float f = pow2_int(fmaxf(k_t - kref, -1000.0f));
+        float hi = s_t * f, lo = e_t * f;
+        for (int o = 16; o > 0; o >>= 1) {
+            const float h2 = __shfl_xor_sync(0xffffffffu, hi, o);
+            const float l2 = __shfl_xor_sync(0xffffffffu, lo, o);
+            float sm, er;
+            two_sum(hi, h2, sm, er);
+            lo = lo + l2 + er;
+            hi = sm;
+        }
+        if (lane == 0) {
+            redh[wid] = hi;
+            redl[wid] = lo;
+        }
+    }
+    // bins of this thread's groups; remember the high ones
+    unsigned long long hmask = 0ull;
+    {
+        int i = 0;
+        for (int g = tid; g < ng; g += NTF, ++i) {
+            const float d = (m - Sketch<DT>::dec(sketch[g])) * a.inv_w;
+            if (d < (float)NBIN) {
+                const int b = (int)d;
+                atomicAdd(&bins[b], 1u);
+                if (b < MASK_BINS && i < MASK_GROUPS) hmask |= 1ull << i;
+            }
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+        double S = 0.0;
+        for (int i = 0; i < NWF; ++i) S += (double)redh[i] + (double)redl[i];
+        s_S = S;
+    }
+    const bool all_in = a.top_p >= 1.0f;
+    if (wid == 0) {
+        constexpr int PER = NBIN / 32;
+        float lb[PER];
+        unsigned cn[PER];
+        float lsum = 0.f;
+        unsigned csum = 0;
+        // a group in bin b carries at least 2^((m - (b+1)T/8) c - kref)
+        const float base2 = ex2(fmaf(m, a.c, -kref));
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            const int b = lane * PER + j;
+            cn[j] = bins[b];
+            lb[j] = (float)cn[j] * ex2(-(float)(b + 1) * (1.4426950408889634f / BIN_PER_T)) * base2;
+            lsum += lb[j];
+            csum += cn[j];
+        }
+        float lpre = lsum;
+        unsigned cpre = csum;
+        for (int o = 1; o < 32; o <<= 1) {
+            const float tt = __shfl_up_sync(0xffffffffu, lpre, o);
+            const unsigned cc = __shfl_up_sync(0xffffffffu, cpre, o);
+            if (lane >= o) {
+                lpre += tt;
+                cpre += cc;
+            }
+        }
+        lpre -= lsum;
+        cpre -= csum;
+        double S = 0.0;  // lane 0 of warp 0 is thread 0, which wrote s_S above
+        if (lane == 0) S = s_S;
+        S = __shfl_sync(0xffffffffu, S, 0);
+        // 1e-4 covers the fp32 sums of the bound and of S
+        const float target = (float)((double)a.top_p * S) * (1.0f + 1e-4f);
+        int hit = -1;
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            lpre += lb[j];
+            cpre += cn[j];
+            const bool okb = all_in ? (cpre >= (unsigned)a.k) : (lpre * (1.0f - 1e-4f) >= target);
+            if (okb && hit < 0) hit = lane * PER + j;
+        }
+        const unsigned bal = __ballot_sync(0xffffffffu, hit >= 0);
+        const int first = bal ? __ffs(bal) - 1 : -1;
+        const int bc = first >= 0 ? __shfl_sync(0xffffffffu, hit, first) : -1;
+        if (lane == 0) {
+            s_bc = bc;
+            s_ncand = 0;
+            s_bigbin = 0;
+        }
+    }
+    __syncthreads();
+    const double S = s_S;
+    const int bc = s_bc;
+    if (!(S > 0.0 && S < 1e300) || !(m < INFINITY) || !(kref < 1e30f)) {
+        nonfinite_row<NTF>(a, r);
+        return;
+    }
+    if (bc < 0) {
+        if (tid == 0) fallback_row(a, r);
+        return;
+    }
+    for (int i = tid; i <= bc; i += NTF) {
+        bins[i] = 0u;
+        bfill[i] = 0u;
+    }
+    __syncthreads();
+
+    // ---- candidates: ids whose bin is <= bc, re-read from their groups ----
+    const float lim = (float)(bc + 1);
+    {
+        const int ngt = (ng - tid + NTF - 1) / NTF;  // groups of this thread
+        const bool use_mask = bc < MASK_BINS && ngt <= MASK_GROUPS;
+        unsigned long long todo = use_mask ? hmask : 0ull;
+        for (int i = 0; use_mask ? (todo != 0ull) : (i < ngt); ++i) {
+            int gi = i;
+            if (use_mask) {
+                gi = __ffsll((long long)todo) - 1;
+                todo &= todo - 1ull;
+            }
+            const int g = tid + gi * NTF;
+            if ((m - Sketch<DT>::dec(sketch[g])) * a.inv_w >= lim) continue;
+#pragma unroll
+            for (int j = 0; j < GC; ++j) {
+                const int cc = g * GC + j;
+                if (cc < nch) {
+                    const uint4 wv = ldg16(row + (size_t)cc * 16);
+#pragma unroll
+                    for (int e = 0; e < EPC; ++e) {
+                        const float v = E::get(wv, e);
+                        const float d = (m - v) * a.inv_w;
+                        if (d < lim) {
+                            const int b = (int)d;
+                            const int pos = atomicAdd(&s_ncand, 1);
+                            if (pos < CAND_CAP_F) {
+                                cand[pos] = order_val(fkey(v), (uint32_t)(cc * EPC + e));
+                                cbin[pos] = (unsigned char)b;
+                                atomicAdd(&bins[b], 1u);
+                            }
+                        }
+                    }
+                }
+            }
+        }
+    }
+    __syncthreads();
+    const int n = s_ncand;
+    if (n > CAND_CAP_F) {
+        if (tid == 0) fallback_row(a, r);
+        return;
+    }
+    // ---- order: bucket by bin (bins descend in value), then inside each bin ----
+    if (wid == 0) {
+        constexpr int PER = NBIN / 32;
+        unsigned cn[PER];
+        unsigned csum = 0, big = 0;
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            const int b = lane * PER + j;
+            cn[j] = b <= bc ? bins[b] : 0u;
+            csum += cn[j];
+            big |= cn[j] > (unsigned)BUCKET_MAX;
+        }
+        unsigned cpre = csum;
+        for (int o = 1; o < 32; o <<= 1) {
+            const unsigned cc = __shfl_up_sync(0xffffffffu, cpre, o);
+            if (lane >= o) cpre += cc;
+        }
+        cpre -= csum;
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            bstart[lane * PER + j] = cpre;
+            cpre += cn[j];
+        }
+        big = __any_sync(0xffffffffu, big);
+        if (lane == 0) s_bigbin = (int)big;
+    }
+    __syncthreads();
+    unsigned long long *ord = sorted;
+    if (!s_bigbin) {
+        for (int i = tid; i < n; i += NTF) {
+            const int b = cbin[i];
+            sorted[bstart[b] + atomicAdd(&bfill[b], 1u)] = cand[i];
+        }
+        __syncthreads();
+        for (int b = tid; b <= bc; b += NTF) {  // insertion sort, descending, inside bin b
+            const int lo = (int)bstart[b], hi = lo + (int)bins[b];
+            for (int i = lo + 1; i < hi; ++i) {
+                const unsigned long long v = sorted[i];
+                int j = i - 1;
+                while (j >= lo && sorted[j] < v) {
+                    sorted[j + 1] = sorted[j];
+                    --j;
+                }
+                sorted[j + 1] = v;
+            }
+        }
+    } else {
+        const int np = next_pow2(n < 2 ? 2 : n);
+        for (int i = n + tid; i < np; i += NTF) cand[i] = 0ull;
+        __syncthreads();
+        bitonic_sort_desc(cand, np);
+        ord = cand;
+    }
+    __syncthreads();
+
+    // ---- nucleus crossing with exact fixed-point prefix sums (warp 0) ----
+    if (wid == 0) {
+        const int per = (n + 31) / 32;
+        const int lo = lane * per, hi = min(n, lo + per);
+        unsigned long long loc = 0ull;
+        for (int i = lo; i < hi; ++i) loc += to_fx(ex2(fmaf(order_value(ord[i]), a.c, -kref)));
+        unsigned long long inc = loc;
+        for (int o = 1; o < 32; o <<= 1) {
+            const unsigned long long tt = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= o) inc += tt;
+        }
+        const unsigned long long ex = inc - loc;
+        int nstar = n - 1;
+        if (!all_in) {
+            const unsigned long long tg = (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
+            int found = INT_MAX;
+            unsigned long long c = ex;
+            for (int i = lo; i < hi; ++i) {
+                c += to_fx(ex2(fmaf(order_value(ord[i]), a.c, -kref)));
+                if (c >= tg) {
+                    found = i;
+                    break;
+                }
+            }
+            const unsigned bal = __ballot_sync(0xffffffffu, found != INT_MAX);
+            nstar = bal ? __shfl_sync(0xffffffffu, found, __ffs(bal) - 1) : INT_MAX;
+        }
+        int L = 0;
+        if (nstar != INT_MAX) L = all_in ? min(n, a.k) : min(nstar + 1, a.k);
+        unsigned long long cN = 0ull, cL = 0ull, c = ex;
+        for (int i = lo; i < hi; ++i) {
+            c += to_fx(ex2(fmaf(order_value(ord[i]), a.c, -kref)));
+            if (i == nstar) cN = c;
+            if (i == L - 1) cL = c;
+        }
+        cN = warp_sum(cN);
+        cL = warp_sum(cL);
+        if (lane == 0) {
+            s_nstar = nstar;
+            s_L = L;
+            s_Snuc_fx = cN;
+            s_cumL_fx = cL;
+            s_cut = (nstar != INT_MAX && !all_in) ? ord[nstar] : 0ull;
+        }
+    }
+    __syncthreads();
+    if (s_nstar == INT_MAX) {  // the candidates carry too little mass: exact path
+        if (tid == 0) fallback_row(a, r);
+        return;
+    }
+    const int L = s_L;
+    const double S_nuc = all_in ? S : (double)s_Snuc_fx / (double)FX_SCALE;
+    const float inv_S = (float)(1.0 / S_nuc);
+    for (int j = tid; j < a.k; j += NTF) {
+        const size_t o = (size_t)r * a.k + j;
+        if (j < L) {
+            const unsigned long long ov = ord[j];
+            a.topk_ids[o] = (int32_t)order_id(ov);
+            a.topk_probs[o] = ex2(fmaf(order_value(ov), a.c, -kref)) * inv_S;
+        } else {
+            a.topk_ids[o] = -1;
+            a.topk_probs[o] = 0.0f;
+        }
+    }
+    if (tid == 0) {
+        const double cumL = (double)s_cumL_fx / (double)FX_SCALE;
+        if (a.k > 0) a.tail[r] = (float)((S_nuc - cumL) / S_nuc);
+        const unsigned long long cut = s_cut;
+        int stt = 0;
+        if (a.K > 0 && iq < a.K) {
+            int accept = 0;
+            if (xb < 0 || xb >= a.V) {
+                stt |= ACES_ROW_BAD_Q;
+            } else {
+                const bool in = all_in ? (zx > -INFINITY) : (order_val(fkey(zx), (uint32_t)xb) >= cut);
+                const double p = in ? (double)ex2(fmaf(zx, a.c, -kref)) / S_nuc : 0.0;
+                if (!(qx > 0.0f)) stt |= ACES_ROW_BAD_Q;
+                else accept = (double)a.u[(size_t)bq * (a.K + 1) + iq] < fmin(1.0, p / (double)qx);
+            }
+            a.ws.acc[(size_t)bq * a.K + iq] = accept;
+        }
+        a.row_status[r] = stt;
+        RowStat rs;
+        rs.kref = kref;
+        rs.c = a.c;
+        rs.S_nuc = S_nuc;
+        rs.cut = cut;
+        rs.flags = all_in ? RS_ALL_IN : 0;
+        rs.pad = 0;
+        a.ws.stats[r] = rs;
+    }
+}
+
+// Chunks per sketch group: the smallest power of two >= 2 that keeps the
+// sketch within SKETCH_CAP groups; 0 when the fast kernel cannot take the row.
+int rows_fast_gc(int dt, int V) {
+    const int nch = (int)((size_t)V * (dt == ACES_BF16 ? 2 : 4) / 16);
+    const int gmax = dt == ACES_BF16 ? 8 : 16;
+    for (int gc = 2; gc <= gmax; gc *= 2)
+        if ((nch + gc - 1) / gc <= SKETCH_CAP) return gc;
+    return 0;
+}
+
+size_t rows_fast_smem(int dt, int gc, int nch) {
+    const size_t skw = dt == ACES_BF16 ? 2 : 4;
+    const int ng = (nch + gc - 1) / gc;
+    size_t sk = align16((size_t)ng * skw);
+    if (sk < (size_t)CAND_CAP_F * 8) sk = (size_t)CAND_CAP_F * 8;
+    return sk + (size_t)CAND_CAP_F * 9;
+}
+
+template <int DT>
+static cudaError_t launch_fast_dt(const RowArgs &a, int gc, size_t smem, cudaStream_t s) {
+    void (*fn)(RowArgs) = nullptr;
+    switch (gc) {
+        case 2: fn = k_rows_fast<DT, 2>; break;
+        case 4: fn = k_rows_fast<DT, 4>; break;
+        case 8: fn = k_rows_fast<DT, 8>; break;
+        case 16:
+            if (DT == ACES_F32) fn = k_rows_fast<ACES_F32, 16>;
+            break;
+        default: break;
+    }
+    if (!fn) return cudaErrorInvalidValue;
+    const cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    fn<<<a.rows, NTF, smem, s>>>(a);
+    return cudaGetLastError();
+}
+
+// one CTA per row (grid = rows); `grid` is unused
+cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, int grid, cudaStream_t s) {
+    (void)grid;
+    return dt == ACES_BF16 ? launch_fast_dt<ACES_BF16>(a, gc, smem, s) : launch_fast_dt<ACES_F32>(a, gc, smem, s);
+}
+
+}  // namespace aces
