@@ -180,6 +180,21 @@ def cache_bytes(B, K, V, S):
 
 
 # ---------------------------------------------------------------------------
+def shard(rank: int, B: int) -> range:
+    """Sequences of this rank: every rank gets its own B sequences (weak scaling)."""
+    return range(rank * B, (rank + 1) * B)
+
+
+def max_over_ranks(x: float, dist=None, device=None) -> float:
+    """The largest x over all ranks (the job's time is its slowest rank's)."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def init_dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -282,7 +297,7 @@ def main():
         import dataclasses
         w = dataclasses.replace(w, B=min(args.B, w.B))
     # host inputs first (spawn pool), this rank's shard of sequences
-    inp = gen.generate_sequences(w, range(rank * w.B, (rank + 1) * w.B), workers=min(16, os.cpu_count() or 1))
+    inp = gen.generate_sequences(w, shard(rank, w.B), workers=min(16, os.cpu_count() or 1))
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
@@ -327,13 +342,6 @@ def main():
             pg.barrier()
         torch.cuda.synchronize()
 
-    def max_over_ranks(x):
-        if pg is None:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        return float(t.item())
-
     for _ in range(args.warmup):
         step()
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
@@ -351,7 +359,7 @@ def main():
             step(evs[i])
         t1.record(stream)
         barrier()
-    ms_total = max_over_ranks(t0.elapsed_time(t1))
+    ms_total = max_over_ranks(t0.elapsed_time(t1), pg, dev)
     ms_step = ms_total / args.steps
     part_ms = {
         "verify_sparsify": statistics.mean(e[0].elapsed_time(e[1]) for e in evs),
@@ -441,7 +449,7 @@ def main():
     for _ in range(e2e_steps):
         e2e_step()
     barrier()
-    e2e_s = max_over_ranks((time.perf_counter() - t) / e2e_steps)
+    e2e_s = max_over_ranks((time.perf_counter() - t) / e2e_steps, pg, dev)
     e2e = {"value": ws * rows / e2e_s, "unit": "rows/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
            "ms_per_step": e2e_s * 1e3}
 
