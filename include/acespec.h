@@ -119,6 +119,37 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
                         aces_stream_t stream);
 
 /*
+ * aces_verify for callers that cannot allocate device memory themselves.
+ * The paper has no counterpart; this is a library convenience.
+ *
+ * Who needs it: a caller with no device allocator on its serving path.
+ * cudaMalloc synchronizes the whole device, which a latency-bound verify loop
+ * cannot afford, and some host runtimes that embed this library own all
+ * device memory.  Such callers cannot supply aces_verify's workspace.
+ *
+ * Same arguments, outputs and errors as aces_verify, without the workspace:
+ * the scratch is a fixed array of ACES_NOALLOC_SCRATCH_BYTES bytes inside the
+ * library, kept on every GPU that loads the library until the process exits.
+ * This call allocates nothing.
+ *   - Size limit: returns ACES_ERR_UNSUPPORTED (nothing launched) when
+ *     aces_workspace_bytes(B, K, V, k) > ACES_NOALLOC_SCRATCH_BYTES, i.e.
+ *     B > 989 at K = 16, B > 1416 at K = 8, B > 1807 at K = 4.
+ *   - Set-up: the first call on each device looks up the array's device
+ *     address (cudaGetSymbolAddress) with that device current; make that
+ *     first call before any stream capture on the device.
+ *   - Sharing: every call on a device uses the same scratch, which keeps the
+ *     last call's contents (each call clears what it needs).  Calls whose
+ *     work overlaps on the GPU race on it: serialize them (one stream, or
+ *     events between streams).
+ */
+#define ACES_NOALLOC_SCRATCH_BYTES (1 << 20)
+aces_status aces_verify_noalloc(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                                const int32_t *draft_tokens, const float *uniforms, int B, int K,
+                                int V, float T, float top_p, int32_t *accept_len,
+                                int32_t *out_token, int k, int32_t *topk_ids, float *topk_probs,
+                                float *tail_mass, int32_t *row_status, aces_stream_t stream);
+
+/*
  * Sparse payload alone for `rows` independent target rows (the COMPRESS of
  * the downlink distribution, Sec. III-B and Sec. V-C): temperature softmax,
  * nucleus, then the first k ids of the nucleus with their renormalised
