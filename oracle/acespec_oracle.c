@@ -23,7 +23,10 @@
  *   3. accept:    a_i = [u_i < min(1, p_i(x~_i) / q_i(x~_i))]
  *   4. pi_b:      first i with a_i = 0, else K           (Sec. III-B)
  *   5. residual:  r = max(0, p_pi - q_pi) (r = p_K when pi = K, the bonus);
- *                 token = smallest j with sum_{x<=j} r_x > u_K * sum r
+ *                 token = smallest j with sum_{x<=j} r_x > u_K * sum r.
+ *                 For a valid draft distribution (q >= 0) r is 0 wherever
+ *                 p = 0, so q is read, and checked for NaN or negative
+ *                 values, only where p > 0.
  *   6. payload:   first k ids of the step-2 order with p > 0, their p, and
  *                 tail = 1 - sum of those p          (Sec. III-B, Sec. V-C)
  *   7. branches:  per depth d, ids != x~_d with q > 0 ordered by
@@ -295,6 +298,7 @@ int orc_verify(const float *z, const float *q, const int32_t *xt, const float *u
                 if (pi < K) {
                     const float *qr = qb + (size_t)pi * V;
                     for (int x = 0; x < V; ++x) {
+                        if (!(pp[x] > 0.0)) { r[x] = 0.0; continue; }  /* max(0, 0 - q), q >= 0 */
                         double qx = (double)qr[x];
                         if (isnan(qx) || qx < 0.0) { bad = 1; break; }
                         double d = pp[x] - qx;

@@ -246,6 +246,22 @@ def test_bad_draft_probability_forces_reject(orc):
     assert out["out_token"][0] == 2                 # residual mass sits where q = 0
 
 
+def test_residual_reads_draft_only_where_target_is_positive(orc):
+    # nucleus of z = [5, 0, 0] at top_p = 0.5 is {0}, so p = (1, 0, 0).  The
+    # draft token 1 has p = 0 and is rejected; r = max(0, p - q) = (0.5, 0, 0)
+    # for any valid q, so token 0 is emitted.  A negative q at id 2 (p = 0)
+    # is never read; a negative q at id 0 makes the residual row invalid.
+    z = np.array([[[5.0, 0.0, 0.0], [0.0, 0.0, 0.0]]] * 2, np.float32)
+    q = np.array([[[0.5, 0.7, -0.2]], [[-0.1, 0.7, 0.4]]], np.float32)
+    xt = np.array([[1], [1]], np.int32)
+    u = np.array([[0.01, 0.999], [0.01, 0.999]], np.float32)
+    out = orc.verify(z, q, xt, u, 1.0, 0.5, 0)
+    assert list(out["accept_len"]) == [0, 0]
+    assert out["row_status"][0, 0] == 0 and out["out_token"][0] == 0
+    assert out["res_sum"][0] == pytest.approx(0.5, abs=1e-15)
+    assert out["row_status"][1, 0] & orc.ROW_BAD_Q and out["out_token"][1] == -1
+
+
 # --------------------------------------------------------------------------
 # step 7-8: branch cache
 
