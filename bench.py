@@ -29,12 +29,17 @@ import sys
 import threading
 import time
 
+import numpy as np
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "verified rows/s and achieved HBM GB/s (fraction of GB300 peak) for verify+sparsify"
 WORKLOAD = "b256_k16_v256000_bf16"
 SWEEP_B = (32, 64, 128, 256)
+# kernels of one step: k_rows_fast, k_rows_general, k_resolve_list,
+# k_resolve_seg, k_resolve_pick (aces_verify), k_cache_build, k_cache_lookup
+KERNELS_PER_STEP = 7
 
 
 # ---------------------------------------------------------------------------
@@ -168,11 +173,29 @@ def profiled_traffic(kernel: str, units: float):
     return e["dram_bytes"] * units / e["units"]
 
 
-def verify_bytes(B, K, V, k, zsize, n_rej):
-    """Algorithmic bytes of one aces_verify call with a payload of k."""
-    rd = B * (K + 1) * V * zsize + n_rej * V * 4 + B * K * 12 + B * 4
+def verify_bytes(B, K, V, k, zsize, n_resid_q):
+    """Algorithmic bytes of one aces_verify call with a payload of k.
+
+    Reads: every logit once, q at the K draft tokens, the draft tokens and
+    the uniforms, and q at the residual row's nucleus ids (n_resid_q floats
+    over the batch; the residual max(0, p - q) is 0 wherever p = 0).
+    Writes: payload, tail and status per row, token and length per sequence.
+    """
+    rd = B * (K + 1) * V * zsize + n_resid_q * 4 + B * K * 12 + B * (K + 1) * 4
     wr = B * (K + 1) * (8 * k + 4) + B * 8 + B * (K + 1) * 4
     return rd + wr
+
+
+def resid_q_count(out, K, k):
+    """q floats the residual step needs: the nucleus of each rejecting
+    sequence's row pi, counted from its payload (a lower bound of the nucleus
+    size when that exceeds k)."""
+    if k == 0:
+        return 0
+    al = out["accept_len"].cpu().numpy()
+    ids = out["topk_ids"].cpu().numpy()
+    rej = np.nonzero(al < K)[0]
+    return int((ids[rej, al[rej]] >= 0).sum())
 
 
 def cache_bytes(B, K, V, S):
@@ -206,8 +229,6 @@ def reference_arm(args, ws, rank):
     """Times the float64 CPU oracle as it stands on a bounded sample."""
     if rank != 0:
         return
-    import numpy as np  # noqa: F401
-
     import gen
     from oracle import oracle as O
     O.build()
@@ -286,7 +307,6 @@ def main():
         reference_arm(args, ws, rank)
         return
 
-    import numpy as np
     import torch
 
     import gen
@@ -371,14 +391,16 @@ def main():
 
     al = out["accept_len"].cpu().numpy()
     n_rej = int((al < K).sum())
+    n_resid_q = resid_q_count(out, K, k)
     fb = int(wsb[:4].view(torch.int32).item())
     peak, peak_kind = measured_peak()
-    vb = verify_bytes(B, K, V, k, zsize, n_rej)
+    vb = verify_bytes(B, K, V, k, zsize, n_resid_q)
     cb = cache_bytes(B, K, V, S)
     parts = {
         "verify_sparsify": {"ms": part_ms["verify_sparsify"], "rows_per_s": rows / (part_ms["verify_sparsify"] * 1e-3),
                             "alg_bytes": vb, "gbs": vb / (part_ms["verify_sparsify"] * 1e-3) / 1e9,
-                            "kernels": ["k_rows_fast", "k_rows_general", "k_resolve"],
+                            "kernels": ["k_rows_fast", "k_rows_general", "k_resolve_list", "k_resolve_seg",
+                                        "k_resolve_pick"],
                             "rows_on_general_path": fb, "rejecting_sequences": n_rej},
         "cache_build": {"ms": part_ms["cache_build"], "alg_bytes": cb,
                         "gbs": cb / (part_ms["cache_build"] * 1e-3) / 1e9, "kernels": ["k_cache_build"]},
@@ -416,8 +438,7 @@ def main():
             e1.record(stream)
             torch.cuda.synchronize()
             ms = e0.elapsed_time(e1) / n
-            nr = int((o2["accept_len"] < K).sum().item())
-            by = verify_bytes(bs, K, V, k, zsize, nr)
+            by = verify_bytes(bs, K, V, k, zsize, resid_q_count(o2, K, k))
             sweep.append({"B": bs, "ms": ms, "rows_per_s": bs * (K + 1) / (ms * 1e-3), "gbs": by / (ms * 1e-3) / 1e9,
                           "frac_of_peak": by / (ms * 1e-3) / 1e9 / peak})
 
@@ -463,7 +484,7 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": config_of(w),
             "roofline": roof, "roofline_verify_sparsify": roof_v, "cpu_baseline": cpu, "e2e": e2e,
-            "gpu_launches": 5 * args.steps, "clocks": clocks.summary(), "parts": parts, "sweep": sweep,
+            "gpu_launches": KERNELS_PER_STEP * args.steps, "clocks": clocks.summary(), "parts": parts, "sweep": sweep,
         }
         print(json.dumps(line), flush=True)
     if pg is not None:

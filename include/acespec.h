@@ -33,6 +33,9 @@
  *     with a finite logit; p is renormalised over the kept set.
  *   - accept: a_i = [u_i < min(1, p_i(x~_i) / q_i(x~_i))]; q_i(x~_i) <= 0,
  *     NaN, or an out-of-range draft token forces a reject (ACES_ROW_BAD_Q).
+ *   - residual: max(0, p - q) is 0 wherever p = 0 for any valid q, so the
+ *     draft row q_pi is read only at ids with p > 0; a NaN or negative q at
+ *     one of those ids marks row pi ACES_ROW_BAD_Q (out_token -1).
  *   - pi_b = first i with a_i = 0, else K.  When pi < K the emitted token is
  *     drawn from norm(max(0, p_pi - q_pi)) (from p_pi if that is all zero);
  *     when pi = K the bonus token is drawn from p_K.  The draw is the
@@ -77,7 +80,8 @@ typedef struct CUstream_st *aces_stream_t;
 
 /*
  * Bytes of device scratch that aces_verify (B sequences, K >= 1) or
- * aces_sparsify (B rows, K = 0) needs.  The caller allocates it, passes it
+ * aces_sparsify (B rows, K = 0) needs (about 4.1 KiB per target row for
+ * aces_verify, under 100 bytes per row for aces_sparsify).  The caller allocates it, passes it
  * to the call and must not use it while the call's work is in flight; it
  * needs no initialisation.  Returns 0 for invalid sizes.
  */
@@ -99,7 +103,8 @@ size_t aces_workspace_bytes(int B, int K, int V, int k);
  *   accept_len    [B]  int32   pi_b, accepted draft tokens (0..K)
  *   out_token     [B]  int32   corrected (pi < K) or bonus (pi = K) token;
  *                              -1 when that row is NONFINITE or its draft
- *                              row holds NaN / negative probabilities
+ *                              row holds a NaN / negative probability at an
+ *                              id with p > 0
  *   row_status    [B, K+1]     int32 ACES_ROW_* bits per row
  * Sparse payload (k >= 1; k = 0 skips it and the three pointers may be NULL):
  *   topk_ids      [B, K+1, k]  int32   first k ids of every row's nucleus
@@ -107,7 +112,9 @@ size_t aces_workspace_bytes(int B, int K, int V, int k);
  *   topk_probs    [B, K+1, k]  float32 their renormalised p, 0 padding
  *   tail_mass     [B, K+1]     float32 1 - sum of the row's topk_probs
  * workspace / workspace_bytes: device scratch of at least
- *   aces_workspace_bytes(B, K, V, k) bytes, 16-byte aligned.
+ *   aces_workspace_bytes(B, K, V, k) bytes, 16-byte aligned.  It includes
+ *   4 KiB per row to keep each row's nucleus (when it has at most 512 ids)
+ *   for the residual draw, which then reads q at those ids only.
  * Limits: 1 <= B, 1 <= K <= ACES_MAX_K, 2 <= V <= ACES_MAX_V,
  *   0 <= k <= min(V, ACES_MAX_TOPK).
  */
@@ -132,8 +139,11 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
  * library, kept on every GPU that loads the library until the process exits.
  * This call allocates nothing.
  *   - Size limit: returns ACES_ERR_UNSUPPORTED (nothing launched) when
- *     aces_workspace_bytes(B, K, V, k) > ACES_NOALLOC_SCRATCH_BYTES, i.e.
- *     B > 989 at K = 16, B > 1416 at K = 8, B > 1807 at K = 4.
+ *     B > 985 at K = 16, B > 1409 at K = 8, B > 1795 at K = 4 (the limit
+ *     does not depend on V or k).  The scratch keeps no nucleus lists
+ *     unless aces_workspace_bytes(B, K, V, k) fits in it (B <= 14 at
+ *     K = 16); without them the residual draw scans its whole row.  The
+ *     results are the same either way.
  *   - Set-up: the first call on each device looks up the array's device
  *     address (cudaGetSymbolAddress) with that device current; make that
  *     first call before any stream capture on the device.

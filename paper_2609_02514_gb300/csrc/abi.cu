@@ -71,14 +71,18 @@ size_t aces_workspace_bytes(int B, int K, int V, int k) {
         return 0;
     long long rows = (long long)B * (K + 1);
     if (rows > INT_MAX / 2) return 0;
-    return ws_bytes((int)rows, B, K);
+    return ws_bytes((int)rows, B, K, true);
 }
 
-aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *draft_probs,
+}  // extern "C"
+
+// Results do not depend on `lists`: without them the residual draw scans its
+// whole row instead of the stored nucleus.
+aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const float *draft_probs,
                         const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
                         float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
                         int32_t *topk_ids, float *topk_probs, float *tail_mass,
-                        int32_t *row_status, void *workspace, size_t workspace_bytes,
+                        int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
                         aces_stream_t stream) {
     if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
     aces_status st = check_rows(target_logits, dt, (long long)B * (K + 1), V, T, top_p, k, false,
@@ -86,7 +90,7 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
     if (st != ACES_OK) return st;
     if (!draft_probs || !draft_tokens || !uniforms || !accept_len || !out_token || !workspace)
         return ACES_ERR_INVALID_ARG;
-    if (!aligned16(workspace) || workspace_bytes < aces_workspace_bytes(B, K, V, k))
+    if (!aligned16(workspace) || workspace_bytes < ws_bytes(B * (K + 1), B, K, lists))
         return ACES_ERR_INVALID_ARG;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     const int rows = B * (K + 1);
@@ -107,7 +111,7 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
     a.topk_probs = topk_probs;
     a.tail = tail_mass;
     a.row_status = row_status;
-    a.ws = ws_carve(workspace, rows, B, K);
+    a.ws = ws_carve(workspace, rows, B, K, lists && top_p < 1.0f);
     a.ng = 0;
     st = run_rows(a, dt, s);
     if (st != ACES_OK) return st;
@@ -126,6 +130,21 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
                      aligned16(draft_probs) && V % 4 == 0;
     if (launch_resolve(r, dt, vec, s) != cudaSuccess) return ACES_ERR_CUDA;
     return ACES_OK;
+}
+
+extern "C" {
+
+aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                        const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                        float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                        int32_t *topk_ids, float *topk_probs, float *tail_mass,
+                        int32_t *row_status, void *workspace, size_t workspace_bytes,
+                        aces_stream_t stream) {
+    if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
+    if (workspace_bytes < aces_workspace_bytes(B, K, V, k)) return ACES_ERR_INVALID_ARG;
+    return verify_impl(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
+                       accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status,
+                       workspace, workspace_bytes, true, stream);
 }
 
 aces_status aces_sparsify(const void *target_logits, aces_dtype dt, int rows, int V, float T,
@@ -154,7 +173,7 @@ aces_status aces_sparsify(const void *target_logits, aces_dtype dt, int rows, in
     a.topk_probs = topk_probs;
     a.tail = tail_mass;
     a.row_status = row_status;
-    a.ws = ws_carve(workspace, rows, rows, 0);
+    a.ws = ws_carve(workspace, rows, rows, 0, false);
     a.ng = 0;
     return run_rows(a, dt, reinterpret_cast<cudaStream_t>(stream));
 }

@@ -4,8 +4,9 @@
 //   k_cache_build   one CTA per (sequence, depth) row of the draft
 //                   distribution: the F_d largest q over ids != x~_d, in
 //                   (q desc, id asc) order, with probability q / (1 - q(x~_d)).
-//                   One HBM pass keeps a sorted top-8 list per thread; the
-//                   block then extracts maxima one at a time.  Fan-outs above
+//                   One HBM pass keeps a sorted top-8 list per thread (one
+//                   32-bit compare per element against the list's 8th best);
+//                   the block then extracts maxima one at a time.  Fan-outs above
 //                   8 repeat the pass below the last extracted order value.
 //   k_cache_lookup  one thread per sequence scanning the F_pi branches.
 #include "common.cuh"
@@ -49,29 +50,31 @@ __global__ void __launch_bounds__(NT) k_cache_build(CacheArgs a) {
             unsigned long long Lst[TOPL];
 #pragma unroll
             for (int i = 0; i < TOPL; ++i) Lst[i] = 0ull;
+            // an element can only enter the list when its raw bits reach those
+            // of the current 8th best (positive floats order like their bits;
+            // negative or NaN q pass this test and are rejected below)
+            uint32_t thr = (uint32_t)(Lst[TOPL - 1] >> 32) & 0x7FFFFFFFu;
+            auto consider = [&](float qv, int x) {
+                if (__float_as_uint(qv) < thr) return;
+                if (!(qv > 0.0f) || x == xd) return;
+                const unsigned long long o = order_val(__float_as_uint(qv) | 0x80000000u, (uint32_t)x);
+                if (o < ub && o > Lst[TOPL - 1]) {
+                    list_insert(Lst, o);
+                    thr = (uint32_t)(Lst[TOPL - 1] >> 32) & 0x7FFFFFFFu;
+                }
+            };
             if (VEC) {
                 const int nch = a.V >> 2;
 #pragma unroll 4
                 for (int cc = tid; cc < nch; cc += NT) {
-                    uint4 w = ldg16(qr + (size_t)cc * 4);
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        float qv = Elem<ACES_F32>::get(w, e);
-                        int x = cc * 4 + e;
-                        if (qv > 0.0f && x != xd) {
-                            unsigned long long o = order_val(__float_as_uint(qv) | 0x80000000u, (uint32_t)x);
-                            if (o < ub) list_insert(Lst, o);
-                        }
-                    }
+                    const uint4 w = ldg16(qr + (size_t)cc * 4);
+                    consider(__uint_as_float(w.x), cc * 4);
+                    consider(__uint_as_float(w.y), cc * 4 + 1);
+                    consider(__uint_as_float(w.z), cc * 4 + 2);
+                    consider(__uint_as_float(w.w), cc * 4 + 3);
                 }
             } else {
-                for (int x = tid; x < a.V; x += NT) {
-                    float qv = __ldg(qr + x);
-                    if (qv > 0.0f && x != xd) {
-                        unsigned long long o = order_val(__float_as_uint(qv) | 0x80000000u, (uint32_t)x);
-                        if (o < ub) list_insert(Lst, o);
-                    }
-                }
+                for (int x = tid; x < a.V; x += NT) consider(__ldg(qr + x), x);
             }
             const int take = min(TOPL, Fd - got);
             bool exhausted = false;

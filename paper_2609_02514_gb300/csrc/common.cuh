@@ -25,7 +25,7 @@ struct RowStat {
     double S_nuc;            // nucleus mass in the same units
     unsigned long long cut;  // order value of the last nucleus id
     int flags;
-    int pad;
+    int nnuc;                // nucleus ids stored in the row's list (-1: none stored)
 };
 static_assert(sizeof(RowStat) == 32, "RowStat layout");
 
@@ -267,6 +267,15 @@ __device__ __forceinline__ bool mbar_wait_bounded(unsigned long long *bar, uint3
     }
     return true;
 }
+// per-thread async copy of 16 bytes, global -> shared (both 16-byte aligned)
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
 // bytes and both addresses must be multiples of 16
 __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, unsigned long long *bar) {
     asm volatile(
@@ -284,22 +293,31 @@ struct SegSum {
     int pad;
 };
 constexpr int NSEG_MAX = 16;
+constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual step
 
 // Workspace layout (all offsets 16-byte aligned)
 struct Workspace {
-    int *fb_count;    // [4]   number of rows handed to the general path
-    RowStat *stats;   // [rows]
-    int *acc;         // [B*K] accept bits
-    int *fb_list;     // [rows]
-    SegSum *seg;      // [B*NSEG_MAX] (verify only)
+    int *fb_count;             // [4]   [0] rows handed to the general path, [1] wait timeouts
+    RowStat *stats;            // [rows]
+    int *acc;                  // [B*K] accept bits
+    int *fb_list;              // [rows]
+    SegSum *seg;               // [B*NSEG_MAX]     (verify only)
+    int *seqdone;              // [B]              (verify only) residual drawn from the list
+    unsigned long long *nuc;   // [rows*NUC_CAP]   (verify with lists) nucleus order values
 };
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
-// rows = B*(K+1) target rows; nseq = B sequences with K draft positions (0 for sparsify)
-__host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K) {
-    return 16 + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
-           align16((size_t)rows * 4) + (K > 0 ? align16((size_t)nseq * NSEG_MAX * sizeof(SegSum)) : 0);
+// rows = B*(K+1) target rows; nseq = B sequences with K draft positions (K = 0: sparsify);
+// lists: keep every row's nucleus (up to NUC_CAP ids) for the residual step
+__host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K, bool lists) {
+    size_t b = 16 + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
+               align16((size_t)rows * 4);
+    if (K > 0) {
+        b += align16((size_t)nseq * NSEG_MAX * sizeof(SegSum)) + align16((size_t)nseq * 4);
+        if (lists) b += (size_t)rows * NUC_CAP * 8;
+    }
+    return b;
 }
-__host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K) {
+__host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K, bool lists) {
     char *p = (char *)base;
     Workspace w;
     w.fb_count = (int *)p;
@@ -310,7 +328,16 @@ __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, in
     p += align16((size_t)nseq * K * 4);
     w.fb_list = (int *)p;
     p += align16((size_t)rows * 4);
-    w.seg = K > 0 ? (SegSum *)p : nullptr;
+    w.seg = nullptr;
+    w.seqdone = nullptr;
+    w.nuc = nullptr;
+    if (K > 0) {
+        w.seg = (SegSum *)p;
+        p += align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
+        w.seqdone = (int *)p;
+        p += align16((size_t)nseq * 4);
+        if (lists) w.nuc = (unsigned long long *)p;
+    }
     return w;
 }
 
@@ -376,7 +403,7 @@ __device__ void nonfinite_row(const RowArgs &a, int r) {
         s.S_nuc = 1.0;
         s.cut = 0;
         s.flags = RS_NONFINITE;
-        s.pad = 0;
+        s.nnuc = -1;
         a.ws.stats[r] = s;
     }
 }
@@ -395,6 +422,14 @@ int rows_fast_gc(int dt, int V);
 cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, int grid, cudaStream_t s);
 cudaError_t launch_rows_general(const RowArgs &a, int dt, bool vec, int direct, int grid, cudaStream_t s);
 cudaError_t launch_resolve(const ResolveArgs &a, int dt, bool vec, cudaStream_t s);
+// aces_verify with a choice: lists = false runs in ws_bytes(rows, B, K, false)
+// bytes of workspace (no nucleus lists; the residual draw scans its row).
+aces_status verify_impl(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                        const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                        float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                        int32_t *topk_ids, float *topk_probs, float *tail_mass,
+                        int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
+                        aces_stream_t stream);
 cudaError_t launch_cache_build(const CacheArgs &a, bool vec, cudaStream_t s);
 cudaError_t launch_cache_lookup(const int32_t *bt, const CacheArgs &a, const int32_t *accept_len,
                                 const int32_t *token, int32_t *slot, cudaStream_t s);

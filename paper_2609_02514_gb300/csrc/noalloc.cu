@@ -52,13 +52,18 @@ extern "C" aces_status aces_verify_noalloc(const void *target_logits, aces_dtype
                                            int32_t *out_token, int k, int32_t *topk_ids, float *topk_probs,
                                            float *tail_mass, int32_t *row_status, aces_stream_t stream) {
     if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
-    const size_t need = aces_workspace_bytes(B, K, V, k);
-    if (need == 0) return ACES_ERR_INVALID_ARG;
-    if (need > (size_t)ACES_NOALLOC_SCRATCH_BYTES) return ACES_ERR_UNSUPPORTED;  // batch too large
+    const size_t full = aces_workspace_bytes(B, K, V, k);
+    if (full == 0) return ACES_ERR_INVALID_ARG;
+    // The nucleus lists (4 KiB per row) only fit for tiny batches; without
+    // them the call needs ws_bytes(rows, B, K, false) bytes.
+    const int rows = B * (K + 1);
+    const bool lists = full <= (size_t)ACES_NOALLOC_SCRATCH_BYTES;
+    if (aces::ws_bytes(rows, B, K, false) > (size_t)ACES_NOALLOC_SCRATCH_BYTES)
+        return ACES_ERR_UNSUPPORTED;  // batch too large
     void *scratch = nullptr;
     const aces_status st = scratch_address(&scratch);
     if (st != ACES_OK) return st;
-    return aces_verify(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p, accept_len,
-                       out_token, k, topk_ids, topk_probs, tail_mass, row_status, scratch,
-                       (size_t)ACES_NOALLOC_SCRATCH_BYTES, stream);
+    return aces::verify_impl(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
+                             accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status, scratch,
+                             (size_t)ACES_NOALLOC_SCRATCH_BYTES, lists, stream);
 }

@@ -36,7 +36,7 @@ constexpr int NWF = NTF / 32;
 constexpr int CAND_CAP_F = 2048;
 constexpr int MASK_GROUPS = 64;     // per-thread groups tracked in the high-group mask
 constexpr int MASK_BINS = 64;       // groups below this bin are remembered per thread
-constexpr int BUCKET_MAX = 32;      // largest bin sorted by insertion
+constexpr int BUCKET_MAX = 32;      // largest bin ranked directly (larger: bitonic sort)
 
 template <int DT> struct Sketch;
 template <> struct Sketch<ACES_F32> {
@@ -216,16 +216,18 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
             redl[wid] = lo;
         }
     }
-    // bins of this thread's groups; remember the high ones
+    // bins of this thread's groups: only groups within MASK_BINS bins of the
+    // max are counted here (and remembered); the rest are counted below
+    // only if the first MASK_BINS bins cannot certify the row
     unsigned long long hmask = 0ull;
     {
         int i = 0;
         for (int g = tid; g < ng; g += NTF, ++i) {
             const float d = (m - Sketch<DT>::dec(sketch[g])) * a.inv_w;
-            if (d < (float)NBIN) {
+            if (d < (float)MASK_BINS) {
                 const int b = (int)d;
                 atomicAdd(&bins[b], 1u);
-                if (b < MASK_BINS && i < MASK_GROUPS) hmask |= 1ull << i;
+                if (i < MASK_GROUPS) hmask |= 1ull << i;
             }
         }
     }
@@ -236,54 +238,65 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         s_S = S;
     }
     const bool all_in = a.top_p >= 1.0f;
-    if (wid == 0) {
-        constexpr int PER = NBIN / 32;
-        float lb[PER];
-        unsigned cn[PER];
-        float lsum = 0.f;
-        unsigned csum = 0;
-        // a group in bin b carries at least 2^((m - (b+1)T/8) c - kref)
-        const float base2 = ex2(fmaf(m, a.c, -kref));
-#pragma unroll
-        for (int j = 0; j < PER; ++j) {
-            const int b = lane * PER + j;
-            cn[j] = bins[b];
-            lb[j] = (float)cn[j] * ex2(-(float)(b + 1) * (1.4426950408889634f / BIN_PER_T)) * base2;
-            lsum += lb[j];
-            csum += cn[j];
-        }
-        float lpre = lsum;
-        unsigned cpre = csum;
-        for (int o = 1; o < 32; o <<= 1) {
-            const float tt = __shfl_up_sync(0xffffffffu, lpre, o);
-            const unsigned cc = __shfl_up_sync(0xffffffffu, cpre, o);
-            if (lane >= o) {
-                lpre += tt;
-                cpre += cc;
+    for (int pass = 0; pass < 2; ++pass) {
+        if (pass == 1) {  // the near bins did not certify: count the far groups too
+            __syncthreads();
+            if (s_bc >= 0) break;
+            for (int g = tid; g < ng; g += NTF) {
+                const float d = (m - Sketch<DT>::dec(sketch[g])) * a.inv_w;
+                if (d >= (float)MASK_BINS && d < (float)NBIN) atomicAdd(&bins[(int)d], 1u);
             }
+            __syncthreads();
         }
-        lpre -= lsum;
-        cpre -= csum;
-        double S = 0.0;  // lane 0 of warp 0 is thread 0, which wrote s_S above
-        if (lane == 0) S = s_S;
-        S = __shfl_sync(0xffffffffu, S, 0);
-        // 1e-4 covers the fp32 sums of the bound and of S
-        const float target = (float)((double)a.top_p * S) * (1.0f + 1e-4f);
-        int hit = -1;
+        if (wid == 0) {
+            constexpr int PER = NBIN / 32;
+            float lb[PER];
+            unsigned cn[PER];
+            float lsum = 0.f;
+            unsigned csum = 0;
+            // a group in bin b carries at least 2^((m - (b+1)T/8) c - kref)
+            const float base2 = ex2(fmaf(m, a.c, -kref));
 #pragma unroll
-        for (int j = 0; j < PER; ++j) {
-            lpre += lb[j];
-            cpre += cn[j];
-            const bool okb = all_in ? (cpre >= (unsigned)a.k) : (lpre * (1.0f - 1e-4f) >= target);
-            if (okb && hit < 0) hit = lane * PER + j;
-        }
-        const unsigned bal = __ballot_sync(0xffffffffu, hit >= 0);
-        const int first = bal ? __ffs(bal) - 1 : -1;
-        const int bc = first >= 0 ? __shfl_sync(0xffffffffu, hit, first) : -1;
-        if (lane == 0) {
-            s_bc = bc;
-            s_ncand = 0;
-            s_bigbin = 0;
+            for (int j = 0; j < PER; ++j) {
+                const int b = lane * PER + j;
+                cn[j] = bins[b];
+                lb[j] = (float)cn[j] * ex2(-(float)(b + 1) * (1.4426950408889634f / BIN_PER_T)) * base2;
+                lsum += lb[j];
+                csum += cn[j];
+            }
+            float lpre = lsum;
+            unsigned cpre = csum;
+            for (int o = 1; o < 32; o <<= 1) {
+                const float tt = __shfl_up_sync(0xffffffffu, lpre, o);
+                const unsigned cc = __shfl_up_sync(0xffffffffu, cpre, o);
+                if (lane >= o) {
+                    lpre += tt;
+                    cpre += cc;
+                }
+            }
+            lpre -= lsum;
+            cpre -= csum;
+            double S = 0.0;  // lane 0 of warp 0 is thread 0, which wrote s_S above
+            if (lane == 0) S = s_S;
+            S = __shfl_sync(0xffffffffu, S, 0);
+            // 1e-4 covers the fp32 sums of the bound and of S
+            const float target = (float)((double)a.top_p * S) * (1.0f + 1e-4f);
+            int hit = -1;
+#pragma unroll
+            for (int j = 0; j < PER; ++j) {
+                lpre += lb[j];
+                cpre += cn[j];
+                const bool okb = all_in ? (cpre >= (unsigned)a.k) : (lpre * (1.0f - 1e-4f) >= target);
+                if (okb && hit < 0) hit = lane * PER + j;
+            }
+            const unsigned bal = __ballot_sync(0xffffffffu, hit >= 0);
+            const int first = bal ? __ffs(bal) - 1 : -1;
+            const int bc = first >= 0 ? __shfl_sync(0xffffffffu, hit, first) : -1;
+            if (lane == 0) {
+                s_bc = bc;
+                s_ncand = 0;
+                s_bigbin = 0;
+            }
         }
     }
     __syncthreads();
@@ -303,28 +316,49 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     }
     __syncthreads();
 
-    // ---- candidates: ids whose bin is <= bc, re-read from their groups ----
+    // ---- candidates: ids whose bin is <= bc, re-read from their groups,
+    // up to four groups' loads in flight per thread ----
     const float lim = (float)(bc + 1);
     {
         const int ngt = (ng - tid + NTF - 1) / NTF;  // groups of this thread
         const bool use_mask = bc < MASK_BINS && ngt <= MASK_GROUPS;
         unsigned long long todo = use_mask ? hmask : 0ull;
-        for (int i = 0; use_mask ? (todo != 0ull) : (i < ngt); ++i) {
-            int gi = i;
-            if (use_mask) {
-                gi = __ffsll((long long)todo) - 1;
-                todo &= todo - 1ull;
+        int next = 0;  // next group index when scanning without the mask
+        constexpr int NB = GC >= 8 ? 1 : 8 / GC;  // eight 16-byte loads in flight
+        for (;;) {
+            int gl[NB];
+            int nb = 0;
+            while (nb < NB) {
+                int gi;
+                if (use_mask) {
+                    if (todo == 0ull) break;
+                    gi = __ffsll((long long)todo) - 1;
+                    todo &= todo - 1ull;
+                } else {
+                    if (next >= ngt) break;
+                    gi = next++;
+                }
+                const int g = tid + gi * NTF;
+                if ((m - Sketch<DT>::dec(sketch[g])) * a.inv_w < lim) gl[nb++] = g;
             }
-            const int g = tid + gi * NTF;
-            if ((m - Sketch<DT>::dec(sketch[g])) * a.inv_w >= lim) continue;
+            if (nb == 0) break;
+            uint4 wv[NB][GC];
 #pragma unroll
-            for (int j = 0; j < GC; ++j) {
-                const int cc = g * GC + j;
-                if (cc < nch) {
-                    const uint4 wv = ldg16(row + (size_t)cc * 16);
+            for (int q = 0; q < NB; ++q)
+#pragma unroll
+                for (int j = 0; j < GC; ++j) {
+                    const int cc = q < nb ? gl[q] * GC + j : nch;
+                    wv[q][j] = cc < nch ? ldg16(row + (size_t)cc * 16) : make_uint4(NI, NI, NI, NI);
+                }
+#pragma unroll
+            for (int q = 0; q < NB; ++q) {
+                if (q >= nb) break;
+#pragma unroll
+                for (int j = 0; j < GC; ++j) {
+                    const int cc = gl[q] * GC + j;
 #pragma unroll
                     for (int e = 0; e < EPC; ++e) {
-                        const float v = E::get(wv, e);
+                        const float v = E::get(wv[q][j], e);
                         const float d = (m - v) * a.inv_w;
                         if (d < lim) {
                             const int b = (int)d;
@@ -373,32 +407,32 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         if (lane == 0) s_bigbin = (int)big;
     }
     __syncthreads();
-    unsigned long long *ord = sorted;
+    // order the candidates into cand[]; sorted[] (the sketch's bytes) then
+    // holds their masses in 2^-40 units
+    unsigned long long *ord = cand;
+    unsigned long long *efx = sorted;
     if (!s_bigbin) {
-        for (int i = tid; i < n; i += NTF) {
+        for (int i = tid; i < n; i += NTF) {  // group by bin
             const int b = cbin[i];
             sorted[bstart[b] + atomicAdd(&bfill[b], 1u)] = cand[i];
         }
         __syncthreads();
-        for (int b = tid; b <= bc; b += NTF) {  // insertion sort, descending, inside bin b
+        for (int p = tid; p < n; p += NTF) {  // place = bin start + rank inside the bin
+            const unsigned long long v = sorted[p];
+            const int b = (int)((m - order_value(v)) * a.inv_w);
             const int lo = (int)bstart[b], hi = lo + (int)bins[b];
-            for (int i = lo + 1; i < hi; ++i) {
-                const unsigned long long v = sorted[i];
-                int j = i - 1;
-                while (j >= lo && sorted[j] < v) {
-                    sorted[j + 1] = sorted[j];
-                    --j;
-                }
-                sorted[j + 1] = v;
-            }
+            int rank = 0;
+            for (int j = lo; j < hi; ++j) rank += sorted[j] > v;
+            cand[lo + rank] = v;
         }
     } else {
         const int np = next_pow2(n < 2 ? 2 : n);
         for (int i = n + tid; i < np; i += NTF) cand[i] = 0ull;
         __syncthreads();
         bitonic_sort_desc(cand, np);
-        ord = cand;
     }
+    __syncthreads();
+    for (int i = tid; i < n; i += NTF) efx[i] = to_fx(ex2(fmaf(order_value(ord[i]), a.c, -kref)));
     __syncthreads();
 
     // ---- nucleus crossing with exact fixed-point prefix sums (warp 0) ----
@@ -406,7 +440,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         const int per = (n + 31) / 32;
         const int lo = lane * per, hi = min(n, lo + per);
         unsigned long long loc = 0ull;
-        for (int i = lo; i < hi; ++i) loc += to_fx(ex2(fmaf(order_value(ord[i]), a.c, -kref)));
+        for (int i = lo; i < hi; ++i) loc += efx[i];
         unsigned long long inc = loc;
         for (int o = 1; o < 32; o <<= 1) {
             const unsigned long long tt = __shfl_up_sync(0xffffffffu, inc, o);
@@ -419,7 +453,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
             int found = INT_MAX;
             unsigned long long c = ex;
             for (int i = lo; i < hi; ++i) {
-                c += to_fx(ex2(fmaf(order_value(ord[i]), a.c, -kref)));
+                c += efx[i];
                 if (c >= tg) {
                     found = i;
                     break;
@@ -432,7 +466,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         if (nstar != INT_MAX) L = all_in ? min(n, a.k) : min(nstar + 1, a.k);
         unsigned long long cN = 0ull, cL = 0ull, c = ex;
         for (int i = lo; i < hi; ++i) {
-            c += to_fx(ex2(fmaf(order_value(ord[i]), a.c, -kref)));
+            c += efx[i];
             if (i == nstar) cN = c;
             if (i == L - 1) cL = c;
         }
@@ -451,6 +485,10 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         if (tid == 0) fallback_row(a, r);
         return;
     }
+    // keep the nucleus (in order) for the residual step when it fits
+    const int nnuc = (a.ws.nuc != nullptr && !all_in && s_nstar + 1 <= NUC_CAP) ? s_nstar + 1 : -1;
+    if (nnuc > 0)
+        for (int i = tid; i < nnuc; i += NTF) a.ws.nuc[(size_t)r * NUC_CAP + i] = ord[i];
     const int L = s_L;
     const double S_nuc = all_in ? S : (double)s_Snuc_fx / (double)FX_SCALE;
     const float inv_S = (float)(1.0 / S_nuc);
@@ -489,7 +527,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         rs.S_nuc = S_nuc;
         rs.cut = cut;
         rs.flags = all_in ? RS_ALL_IN : 0;
-        rs.pad = 0;
+        rs.nnuc = nnuc;
         a.ws.stats[r] = rs;
     }
 }

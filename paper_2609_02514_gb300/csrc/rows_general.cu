@@ -21,25 +21,30 @@ __device__ void finish_row(const RowArgs &a, int r, const char *row, float kref,
                            unsigned long long cut, int flags, const unsigned long long *sorted,
                            int L, double *redd) {
     const int tid = threadIdx.x;
-    double loc = 0.0;
+    // same formulas as the fast row kernel, so a row gets bit-identical
+    // outputs whichever kernel finishes it: p = e * (float)(1/S_nuc), and the
+    // tail from the exact fixed-point sum of the payload masses
+    const float inv_S = (float)(1.0 / S_nuc);
+    unsigned long long loc = 0ull;
     if (a.k > 0) {
         for (int j = tid; j < a.k; j += NT) {
             size_t o = (size_t)r * a.k + j;
             if (j < L) {
                 unsigned long long ov = sorted[j];
                 float e = ex2(fmaf(order_value(ov), a.c, -kref));
-                loc += (double)e;
+                loc += to_fx(e);
                 a.topk_ids[o] = (int32_t)order_id(ov);
-                a.topk_probs[o] = (float)((double)e / S_nuc);
+                a.topk_probs[o] = e * inv_S;
             } else {
                 a.topk_ids[o] = -1;
                 a.topk_probs[o] = 0.0f;
             }
         }
     }
-    double tot = block_reduce(loc, redd, SumD());
+    __shared__ unsigned long long s_redl[NWARP];
+    const unsigned long long tot = block_reduce(loc, s_redl, SumU64());
     if (tid != 0) return;
-    if (a.k > 0) a.tail[r] = (float)((S_nuc - tot) / S_nuc);
+    if (a.k > 0) a.tail[r] = (float)((S_nuc - (double)tot / (double)FX_SCALE) / S_nuc);
     int st = 0;
     if (a.K > 0) {
         int b = r / (a.K + 1), i = r % (a.K + 1);
@@ -70,7 +75,7 @@ __device__ void finish_row(const RowArgs &a, int r, const char *row, float kref,
     s.S_nuc = S_nuc;
     s.cut = cut;
     s.flags = flags;
-    s.pad = 0;
+    s.nnuc = -1;  // the residual step scans the row
     a.ws.stats[r] = s;
 }
 

@@ -218,6 +218,57 @@ def test_nonfinite_rows_and_bad_drafts(A, orc):
     assert res["checked_seqs"] >= 6
 
 
+def test_residual_draw_with_and_without_stored_nucleus(A, orc):
+    # Per-sequence logit scales give residual rows whose nucleus is a few ids
+    # (drawn from the stored list) up to thousands of ids (drawn by the scan).
+    w = gen.make_workload(24, 4, 8192, "f32", T=1.0, top_p=0.9, k=8, seed=22)
+    inp = gen.generate(w)
+    scale = np.geomspace(0.05, 8.0, w.B).astype(np.float32)
+    inp["z"] = (inp["z"] * scale[:, None, None]).astype(np.float32)
+    g, o, res = check_all(A, orc, inp, w)
+    pi = o["accept_len"]
+    nres = o["n_nuc"][np.arange(w.B), pi]
+    assert (nres <= 512).sum() >= 4 and (nres > 512).sum() >= 4, nres
+    assert res["checked_seqs"] >= 20
+
+
+def test_draft_probability_read_only_inside_the_nucleus(A, orc):
+    # Residual row 0 of every sequence: the draft token has p = 0 (rejected).
+    # A negative q outside the residual row's nucleus is never read; inside
+    # it marks the row ACES_ROW_BAD_Q and the token is -1.
+    w = gen.make_workload(6, 2, 4096, "f32", T=1.0, top_p=0.5, k=8, seed=24)
+    inp = gen.generate(w)
+    z, q, xt, u = (inp[key].copy() for key in ("z", "q", "xt", "u"))
+    for b in range(w.B):
+        order = np.lexsort((np.arange(w.V), -z[b, 0].astype(np.float64)))
+        xt[b, 0] = order[-1]                       # lowest logit: outside the nucleus
+        q[b, 0, order[-1]] = max(q[b, 0, order[-1]], 1e-3)
+        if b % 2 == 0:
+            q[b, 0, order[-2]] = -0.25             # outside the nucleus
+        else:
+            q[b, 0, order[0]] = -0.25              # the top id, inside
+    inp2 = dict(z=z, q=q, xt=xt, u=u)
+    for tp in (0.5, 1.0):                          # stored list / full-row scan
+        if tp == 1.0:
+            z2 = z.copy()
+            for b in range(w.B):
+                order = np.lexsort((np.arange(w.V), -z[b, 0].astype(np.float64)))
+                z2[b, 0, order[-2]] = -np.inf      # p = 0 there at top_p = 1 too
+                z2[b, 0, order[-1]] = -np.inf
+            inp2 = dict(z=z2, q=q, xt=xt, u=u)
+        g = run_gpu(A, inp2, gen.make_workload(6, 2, 4096, "f32", T=1.0, top_p=tp, k=8, seed=24), 8)
+        o = orc.verify(inp2["z"], q, xt, u, 1.0, tp, 8)
+        assert (o["accept_len"] == 0).all()
+        for b in range(w.B):
+            assert g["accept_len"][b] == 0
+            assert g["row_status"][b, 0] == o["row_status"][b, 0]
+            assert g["out_token"][b] == o["out_token"][b]
+            if b % 2 == 0:
+                assert g["row_status"][b, 0] == 0 and g["out_token"][b] >= 0
+            else:
+                assert g["row_status"][b, 0] & 2 and g["out_token"][b] == -1
+
+
 def test_top_p_boundary_cases(A, orc):
     w, inp = _edge_inputs()
     for top_p in (1e-6, 0.5, 0.999999, 1.0):
