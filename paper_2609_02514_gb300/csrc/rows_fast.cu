@@ -2,25 +2,32 @@
 // packaging of the target distribution; Sec. V-C: compact payload; the
 // acceptance rule is the modified rejection sampling of Sec. II-A).
 //
-// One CTA of 256 threads per target row r = b*(K+1)+i, four CTAs per SM, so
-// that the short per-row epilogue of one row overlaps the HBM stream of the
-// others.
+// One CTA of 256 threads per target row r = b*(K+1)+i, three CTAs per SM
+// (up to 80 registers per thread, so that every thread keeps eight 16-byte
+// loads in flight), so that the per-row epilogue of one row overlaps the
+// HBM stream of the others.
 //
-//   pass 1   every logit is read once from HBM with 16-byte loads (four in
+//   pass 1   every logit is read once from HBM with 16-byte loads (eight in
 //            flight per thread): an online exp-sum in log2 units against an
-//            integer reference k_t = ceil(max z * log2(e)/T) (one FFMA and
-//            one ex2 per logit, rescales are exact powers of two), and the
-//            max of every group of 8*GC consecutive logits into a sketch.
-//   certify  groups are binned by (m - gmax) / (T/8); one max per group is
-//            a lower bound of the mass above a bin edge, so the first bin
-//            whose bound reaches top_p * S proves that the nucleus lies
-//            above that edge (for top_p = 1: the first bin holding k groups
-//            proves the top k lie above it).  Rows the sketch cannot certify
-//            go to the exact general kernel.
-//   select   ids above the edge are re-read (their groups only), bucketed by
-//            bin and ordered inside each bin by the 64-bit (logit, id)
-//            order; the nucleus crossing is found with exact fixed-point
-//            prefix sums in one warp.
+//            integer reference k_t = ceil(max z * log2(e)/T) (one paired
+//            FFMA per two logits, one ex2 per logit, rescales are exact
+//            powers of two), the two largest group maxima per thread, and the
+//            max of every group of GC consecutive 16-byte chunks into a sketch.
+//   certify  group maxima are binned by (m - gmax) / (T/8); one max per
+//            group is a lower bound of the mass above a bin edge, so the
+//            first bin whose bound reaches top_p * S proves that the nucleus
+//            lies above that edge (for top_p = 1: the first bin holding k
+//            groups proves the top k lie above it).  First tier: the two
+//            largest group maxima of every thread, kept in registers during
+//            pass 1; second tier (only when the first cannot certify): every
+//            group of the sketch.  Rows neither can certify go to the exact
+//            general kernel.
+//   select   a binary search turns the edge into a key threshold; groups
+//            whose sketch key reaches it are listed, re-read (one 16-byte
+//            chunk per thread), and their ids above the threshold ordered by
+//            the 64-bit (logit, id) order (direct ranking up to 512 ids,
+//            bitonic sort above); the nucleus crossing is found with exact
+//            fixed-point prefix sums in one warp.
 //   finish   payload (first k of the nucleus), tail mass, accept test of the
 //            draft token at this position, per-row state for the resolve
 //            kernels.
@@ -34,9 +41,7 @@ namespace aces {
 constexpr int NTF = 256;
 constexpr int NWF = NTF / 32;
 constexpr int CAND_CAP_F = 2048;
-constexpr int MASK_GROUPS = 64;     // per-thread groups tracked in the high-group mask
-constexpr int MASK_BINS = 64;       // groups below this bin are remembered per thread
-constexpr int BUCKET_MAX = 32;      // largest bin ranked directly (larger: bitonic sort)
+constexpr int RANK_MAX = 512;       // candidates ordered by direct ranking (more: bitonic sort)
 
 template <int DT> struct Sketch;
 template <> struct Sketch<ACES_F32> {
@@ -83,23 +88,61 @@ __device__ __forceinline__ float group_max(const uint4 (&w)[GC]) {
     }
 }
 
-// sum over the group of 2^(z*c - k)
+// Paired fp32 arithmetic (one instruction for two lanes of a 64-bit register
+// pair; each lane rounds exactly like the scalar operation).
+__device__ __forceinline__ unsigned long long pack2(float lo, float hi) {
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void unpack2(unsigned long long v, float &lo, float &hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ unsigned long long ffma2(unsigned long long a, unsigned long long b,
+                                                    unsigned long long c) {
+    unsigned long long d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+__device__ __forceinline__ unsigned long long fadd2(unsigned long long a, unsigned long long b) {
+    unsigned long long d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+// (2^(lo*c + nk), 2^(hi*c + nk)) for a pair of logits
+__device__ __forceinline__ unsigned long long ex2_pair(unsigned long long z2, unsigned long long c2,
+                                                       unsigned long long nk2) {
+    float lo, hi;
+    unpack2(ffma2(z2, c2, nk2), lo, hi);
+    return pack2(ex2(lo), ex2(hi));
+}
+
+// sum over the group of 2^(z*c - k), two logits per instruction
 template <int DT, int GC>
 __device__ __forceinline__ float group_expsum(const uint4 (&w)[GC], float c, float nk) {
-    using E = Elem<DT>;
-    float gs = 0.f;
+    const unsigned long long c2 = pack2(c, c), nk2 = pack2(nk, nk);
+    unsigned long long acc = 0ull;
 #pragma unroll
     for (int j = 0; j < GC; ++j) {
-        float cs[E::EPC];
+        unsigned long long s;
+        if (DT == ACES_BF16) {
+            const uint32_t wd[4] = {w[j].x, w[j].y, w[j].z, w[j].w};
+            unsigned long long p[4];
 #pragma unroll
-        for (int e = 0; e < E::EPC; ++e) cs[e] = ex2(fmaf(E::get(w[j], e), c, nk));
-#pragma unroll
-        for (int wdt = 1; wdt < E::EPC; wdt <<= 1)
-#pragma unroll
-            for (int e = 0; e < E::EPC; e += 2 * wdt) cs[e] += cs[e + wdt];
-        gs += cs[0];
+            for (int q = 0; q < 4; ++q)
+                p[q] = ex2_pair(pack2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xFFFF0000u)),
+                                c2, nk2);
+            s = fadd2(fadd2(p[0], p[1]), fadd2(p[2], p[3]));
+        } else {
+            const unsigned long long p0 = ex2_pair(pack2(__uint_as_float(w[j].x), __uint_as_float(w[j].y)), c2, nk2);
+            const unsigned long long p1 = ex2_pair(pack2(__uint_as_float(w[j].z), __uint_as_float(w[j].w)), c2, nk2);
+            s = fadd2(p0, p1);
+        }
+        acc = j == 0 ? s : fadd2(acc, s);
     }
-    return gs;
+    float a, b;
+    unpack2(acc, a, b);
+    return a + b;
 }
 
 __device__ __forceinline__ void fallback_row(const RowArgs &a, int r) {
@@ -108,7 +151,7 @@ __device__ __forceinline__ void fallback_row(const RowArgs &a, int r) {
 }
 
 template <int DT, int GC>
-__global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
+__global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
     using E = Elem<DT>;
     using SK = typename Sketch<DT>::T;
     constexpr int EPC = E::EPC;
@@ -119,13 +162,12 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
                                 ? align16((size_t)ng * sizeof(SK)) : (size_t)CAND_CAP_F * 8;
     unsigned long long *sorted = reinterpret_cast<unsigned long long *>(smem);  // after collection
     unsigned long long *cand = reinterpret_cast<unsigned long long *>(smem + sk_bytes);
-    unsigned char *cbin = smem + sk_bytes + (size_t)CAND_CAP_F * 8;
 
     __shared__ uint32_t bins[NBIN];
-    __shared__ uint32_t bstart[NBIN], bfill[NBIN];
     __shared__ float redf[NWF], redk[NWF], redh[NWF], redl[NWF];
-    __shared__ int s_ncand, s_bc, s_nstar, s_L, s_bigbin;
-    __shared__ double s_S;
+    __shared__ int s_ncand, s_ngl, s_bc, s_nstar, s_L;
+    __shared__ double s_S, s_Snuc;
+    __shared__ float s_inv_S;
     __shared__ unsigned long long s_cut, s_Snuc_fx, s_cumL_fx;
 
     const int r = blockIdx.x;
@@ -144,7 +186,9 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
 
     // ---- pass 1 ----
     float k_t = -1e30f, m_t = -INFINITY, s_t = 0.f, e_t = 0.f;
-    constexpr int GPI = GC >= 4 ? 1 : 2;  // groups per iteration: four 16-byte loads in flight
+    float t1 = -INFINITY, t2 = -INFINITY;  // this thread's two largest group maxima
+    // groups per iteration: eight 16-byte loads in flight per thread
+    constexpr int GPI = GC >= 8 ? 1 : 8 / GC;
     for (int g0 = tid; g0 < ng; g0 += NTF * GPI) {
         uint4 w[GPI][GC];
 #pragma unroll
@@ -161,6 +205,10 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
             const int g = g0 + h * NTF;
             const float gm = group_max<DT, GC>(w[h]);
             m_t = fmaxf(m_t, gm);
+            if (gm > t2) {
+                t2 = fminf(gm, t1);
+                t1 = fmaxf(gm, t1);
+            }
             const float gk = gm * a.c;
             if (gk > k_t) {
                 const float nk = ceilf(gk);
@@ -216,20 +264,12 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
             redl[wid] = lo;
         }
     }
-    // bins of this thread's groups: only groups within MASK_BINS bins of the
-    // max are counted here (and remembered); the rest are counted below
-    // only if the first MASK_BINS bins cannot certify the row
-    unsigned long long hmask = 0ull;
+    // first tier: bins of the 2 * NTF largest group maxima (two per thread);
+    // they carry a lower bound of the mass above every bin edge as well
     {
-        int i = 0;
-        for (int g = tid; g < ng; g += NTF, ++i) {
-            const float d = (m - Sketch<DT>::dec(sketch[g])) * a.inv_w;
-            if (d < (float)MASK_BINS) {
-                const int b = (int)d;
-                atomicAdd(&bins[b], 1u);
-                if (i < MASK_GROUPS) hmask |= 1ull << i;
-            }
-        }
+        const float d1 = (m - t1) * a.inv_w, d2 = (m - t2) * a.inv_w;
+        if (d1 < (float)NBIN) atomicAdd(&bins[(int)d1], 1u);
+        if (d2 < (float)NBIN) atomicAdd(&bins[(int)d2], 1u);
     }
     __syncthreads();
     if (tid == 0) {
@@ -239,12 +279,14 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     }
     const bool all_in = a.top_p >= 1.0f;
     for (int pass = 0; pass < 2; ++pass) {
-        if (pass == 1) {  // the near bins did not certify: count the far groups too
+        if (pass == 1) {  // second tier: every group of the sketch
             __syncthreads();
             if (s_bc >= 0) break;
+            for (int i = tid; i < NBIN; i += NTF) bins[i] = 0u;
+            __syncthreads();
             for (int g = tid; g < ng; g += NTF) {
                 const float d = (m - Sketch<DT>::dec(sketch[g])) * a.inv_w;
-                if (d >= (float)MASK_BINS && d < (float)NBIN) atomicAdd(&bins[(int)d], 1u);
+                if (d < (float)NBIN) atomicAdd(&bins[(int)d], 1u);
             }
             __syncthreads();
         }
@@ -295,7 +337,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
             if (lane == 0) {
                 s_bc = bc;
                 s_ncand = 0;
-                s_bigbin = 0;
+                s_ngl = 0;
             }
         }
     }
@@ -310,68 +352,82 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         if (tid == 0) fallback_row(a, r);
         return;
     }
-    for (int i = tid; i <= bc; i += NTF) {
-        bins[i] = 0u;
-        bfill[i] = 0u;
-    }
-    __syncthreads();
-
-    // ---- candidates: ids whose bin is <= bc, re-read from their groups,
-    // up to four groups' loads in flight per thread ----
+    // ---- candidates: every id whose bin is <= bc.  Bins are monotone in the
+    // order key, so a binary search finds the smallest sketch key in a bin
+    // <= bc and the scans below select exactly those ids by integer compares.
     const float lim = (float)(bc + 1);
+    uint32_t thr;
     {
-        const int ngt = (ng - tid + NTF - 1) / NTF;  // groups of this thread
-        const bool use_mask = bc < MASK_BINS && ngt <= MASK_GROUPS;
-        unsigned long long todo = use_mask ? hmask : 0ull;
-        int next = 0;  // next group index when scanning without the mask
-        constexpr int NB = GC >= 8 ? 1 : 8 / GC;  // eight 16-byte loads in flight
-        for (;;) {
-            int gl[NB];
-            int nb = 0;
-            while (nb < NB) {
-                int gi;
-                if (use_mask) {
-                    if (todo == 0ull) break;
-                    gi = __ffsll((long long)todo) - 1;
-                    todo &= todo - 1ull;
-                } else {
-                    if (next >= ngt) break;
-                    gi = next++;
-                }
-                const int g = tid + gi * NTF;
-                if ((m - Sketch<DT>::dec(sketch[g])) * a.inv_w < lim) gl[nb++] = g;
+        uint32_t lo = 0, hi = Sketch<DT>::enc(fkey(m));  // the max itself is in bin 0
+        while (lo < hi) {
+            const uint32_t mid = lo + ((hi - lo) >> 1);
+            if ((m - Sketch<DT>::dec((SK)mid)) * a.inv_w < lim) hi = mid;
+            else lo = mid + 1;
+        }
+        thr = hi;
+    }
+    const uint32_t thr_key = DT == ACES_BF16 ? thr << 16 : thr;  // for 32-bit element keys
+    // groups holding candidates: the sketch is scanned 16 bytes at a time
+    // with packed compares; hits are listed in cand[] (free until ranking)
+    int *glist = reinterpret_cast<int *>(cand);
+    {
+        constexpr int SPW = 16 / sizeof(SK);  // sketch entries per 16-byte word
+        const int nw = (ng + SPW - 1) / SPW;
+        const uint4 *sk4 = reinterpret_cast<const uint4 *>(sketch);
+        for (int i = tid; i < nw; i += NTF) {
+            const uint4 wd = sk4[i];
+            const uint32_t x[4] = {wd.x, wd.y, wd.z, wd.w};
+            unsigned any = 0;
+            if (DT == ACES_BF16) {
+                const uint32_t t2x = thr * 0x00010001u;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) any |= __vcmpgeu2(x[q], t2x);
+            } else {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) any |= x[q] >= thr;
             }
-            if (nb == 0) break;
-            uint4 wv[NB][GC];
+            if (any) {
 #pragma unroll
-            for (int q = 0; q < NB; ++q)
-#pragma unroll
-                for (int j = 0; j < GC; ++j) {
-                    const int cc = q < nb ? gl[q] * GC + j : nch;
-                    wv[q][j] = cc < nch ? ldg16(row + (size_t)cc * 16) : make_uint4(NI, NI, NI, NI);
-                }
-#pragma unroll
-            for (int q = 0; q < NB; ++q) {
-                if (q >= nb) break;
-#pragma unroll
-                for (int j = 0; j < GC; ++j) {
-                    const int cc = gl[q] * GC + j;
-#pragma unroll
-                    for (int e = 0; e < EPC; ++e) {
-                        const float v = E::get(wv[q][j], e);
-                        const float d = (m - v) * a.inv_w;
-                        if (d < lim) {
-                            const int b = (int)d;
-                            const int pos = atomicAdd(&s_ncand, 1);
-                            if (pos < CAND_CAP_F) {
-                                cand[pos] = order_val(fkey(v), (uint32_t)(cc * EPC + e));
-                                cbin[pos] = (unsigned char)b;
-                                atomicAdd(&bins[b], 1u);
-                            }
-                        }
+                for (int e = 0; e < SPW; ++e) {
+                    const int g = i * SPW + e;
+                    if (g < ng && (uint32_t)sketch[g] >= thr) {
+                        const int pos = atomicAdd(&s_ngl, 1);
+                        if (pos < CAND_CAP_F) glist[pos] = g;
                     }
                 }
             }
+        }
+    }
+    __syncthreads();
+    const int ngl = s_ngl;
+    if (ngl > CAND_CAP_F) {  // every listed group holds a candidate: too many
+        if (tid == 0) fallback_row(a, r);
+        return;
+    }
+    // re-read the listed groups, one 16-byte chunk per thread and round;
+    // candidates go to sorted[] (the sketch is no longer needed)
+    unsigned long long *cv = sorted;
+    {
+        const int nck = ngl * GC;
+        for (int c0 = 0; c0 < nck; c0 += 2 * NTF) {
+            uint4 wv[2];
+            int cc[2];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int c = c0 + h * NTF + tid;
+                cc[h] = c < nck ? glist[c / GC] * GC + c % GC : nch;
+                wv[h] = cc[h] < nch ? ldg16(row + (size_t)cc[h] * 16) : make_uint4(NI, NI, NI, NI);
+            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int e = 0; e < EPC; ++e) {
+                    const uint32_t key = fkey(E::get(wv[h], e));
+                    if (cc[h] < nch && key >= thr_key) {
+                        const int pos = atomicAdd(&s_ncand, 1);
+                        if (pos < CAND_CAP_F) cv[pos] = order_val(key, (uint32_t)(cc[h] * EPC + e));
+                    }
+                }
         }
     }
     __syncthreads();
@@ -380,59 +436,27 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         if (tid == 0) fallback_row(a, r);
         return;
     }
-    // ---- order: bucket by bin (bins descend in value), then inside each bin ----
-    if (wid == 0) {
-        constexpr int PER = NBIN / 32;
-        unsigned cn[PER];
-        unsigned csum = 0, big = 0;
-#pragma unroll
-        for (int j = 0; j < PER; ++j) {
-            const int b = lane * PER + j;
-            cn[j] = b <= bc ? bins[b] : 0u;
-            csum += cn[j];
-            big |= cn[j] > (unsigned)BUCKET_MAX;
-        }
-        unsigned cpre = csum;
-        for (int o = 1; o < 32; o <<= 1) {
-            const unsigned cc = __shfl_up_sync(0xffffffffu, cpre, o);
-            if (lane >= o) cpre += cc;
-        }
-        cpre -= csum;
-#pragma unroll
-        for (int j = 0; j < PER; ++j) {
-            bstart[lane * PER + j] = cpre;
-            cpre += cn[j];
-        }
-        big = __any_sync(0xffffffffu, big);
-        if (lane == 0) s_bigbin = (int)big;
-    }
-    __syncthreads();
-    // order the candidates into cand[]; sorted[] (the sketch's bytes) then
-    // holds their masses in 2^-40 units
+    // ---- order the candidates (descending order value) into ord[] (the
+    // cand[] bytes), their masses in 2^-40 units into efx[] ----
     unsigned long long *ord = cand;
-    unsigned long long *efx = sorted;
-    if (!s_bigbin) {
-        for (int i = tid; i < n; i += NTF) {  // group by bin
-            const int b = cbin[i];
-            sorted[bstart[b] + atomicAdd(&bfill[b], 1u)] = cand[i];
-        }
-        __syncthreads();
-        for (int p = tid; p < n; p += NTF) {  // place = bin start + rank inside the bin
-            const unsigned long long v = sorted[p];
-            const int b = (int)((m - order_value(v)) * a.inv_w);
-            const int lo = (int)bstart[b], hi = lo + (int)bins[b];
+    unsigned long long *efx;
+    if (n <= RANK_MAX) {  // rank of each candidate by direct count
+        efx = sorted + RANK_MAX;
+        for (int i = tid; i < n; i += NTF) {
+            const unsigned long long v = cv[i];
             int rank = 0;
-            for (int j = lo; j < hi; ++j) rank += sorted[j] > v;
-            cand[lo + rank] = v;
+            for (int j = 0; j < n; ++j) rank += cv[j] > v;
+            ord[rank] = v;
+            efx[rank] = to_fx(ex2(fmaf(order_value(v), a.c, -kref)));
         }
     } else {
-        const int np = next_pow2(n < 2 ? 2 : n);
-        for (int i = n + tid; i < np; i += NTF) cand[i] = 0ull;
+        const int np = next_pow2(n);
+        for (int i = tid; i < np; i += NTF) ord[i] = i < n ? cv[i] : 0ull;
         __syncthreads();
-        bitonic_sort_desc(cand, np);
+        bitonic_sort_desc(ord, np);
+        efx = sorted;
+        for (int i = tid; i < n; i += NTF) efx[i] = to_fx(ex2(fmaf(order_value(ord[i]), a.c, -kref)));
     }
-    __syncthreads();
-    for (int i = tid; i < n; i += NTF) efx[i] = to_fx(ex2(fmaf(order_value(ord[i]), a.c, -kref)));
     __syncthreads();
 
     // ---- nucleus crossing with exact fixed-point prefix sums (warp 0) ----
@@ -477,6 +501,9 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
             s_L = L;
             s_Snuc_fx = cN;
             s_cumL_fx = cL;
+            const double sn = all_in ? S : (double)cN / (double)FX_SCALE;
+            s_Snuc = sn;
+            s_inv_S = (float)(1.0 / sn);  // one fp64 divide per row
             s_cut = (nstar != INT_MAX && !all_in) ? ord[nstar] : 0ull;
         }
     }
@@ -490,8 +517,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     if (nnuc > 0)
         for (int i = tid; i < nnuc; i += NTF) a.ws.nuc[(size_t)r * NUC_CAP + i] = ord[i];
     const int L = s_L;
-    const double S_nuc = all_in ? S : (double)s_Snuc_fx / (double)FX_SCALE;
-    const float inv_S = (float)(1.0 / S_nuc);
+    const float inv_S = s_inv_S;
     for (int j = tid; j < a.k; j += NTF) {
         const size_t o = (size_t)r * a.k + j;
         if (j < L) {
@@ -504,6 +530,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         }
     }
     if (tid == 0) {
+        const double S_nuc = s_Snuc;
         const double cumL = (double)s_cumL_fx / (double)FX_SCALE;
         if (a.k > 0) a.tail[r] = (float)((S_nuc - cumL) / S_nuc);
         const unsigned long long cut = s_cut;
@@ -536,7 +563,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
 // sketch within SKETCH_CAP groups; 0 when the fast kernel cannot take the row.
 int rows_fast_gc(int dt, int V) {
     const int nch = (int)((size_t)V * (dt == ACES_BF16 ? 2 : 4) / 16);
-    const int gmax = dt == ACES_BF16 ? 8 : 16;
+    const int gmax = 8;  // 16 chunks per group would not fit the register budget
     for (int gc = 2; gc <= gmax; gc *= 2)
         if ((nch + gc - 1) / gc <= SKETCH_CAP) return gc;
     return 0;
@@ -547,7 +574,7 @@ size_t rows_fast_smem(int dt, int gc, int nch) {
     const int ng = (nch + gc - 1) / gc;
     size_t sk = align16((size_t)ng * skw);
     if (sk < (size_t)CAND_CAP_F * 8) sk = (size_t)CAND_CAP_F * 8;
-    return sk + (size_t)CAND_CAP_F * 9;
+    return sk + (size_t)CAND_CAP_F * 8;
 }
 
 template <int DT>
@@ -557,9 +584,6 @@ static cudaError_t launch_fast_dt(const RowArgs &a, int gc, size_t smem, cudaStr
         case 2: fn = k_rows_fast<DT, 2>; break;
         case 4: fn = k_rows_fast<DT, 4>; break;
         case 8: fn = k_rows_fast<DT, 8>; break;
-        case 16:
-            if (DT == ACES_F32) fn = k_rows_fast<ACES_F32, 16>;
-            break;
         default: break;
     }
     if (!fn) return cudaErrorInvalidValue;
