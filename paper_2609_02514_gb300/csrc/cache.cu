@@ -4,35 +4,38 @@
 //   k_cache_build   one CTA per (sequence, depth) row of the draft
 //                   distribution: the F_d largest q over ids != x~_d, in
 //                   (q desc, id asc) order, with probability q / (1 - q(x~_d)).
-//                   One HBM pass keeps a sorted top-8 list per thread (one
-//                   32-bit compare per element against the list's 8th best);
-//                   the block then extracts maxima one at a time.  Fan-outs above
-//                   8 repeat the pass below the last extracted order value.
+//                   One HBM pass keeps a sorted top-TOPL list per thread
+//                   (TOPL = 4 when every F_d <= 4, else 8), filtered by one
+//                   integer max and compare per four values against the raw
+//                   bits of the list's last entry; the block then extracts
+//                   maxima one at a time.  Fan-outs above TOPL repeat the
+//                   pass below the last extracted order value.
 //   k_cache_lookup  one thread per sequence scanning the F_pi branches.
 #include "common.cuh"
 
 namespace aces {
 
 
-constexpr int TOPL = 8;  // per-thread list length
+constexpr int NTC = 256;  // threads per row
+constexpr int CLD = 8;    // 16-byte loads in flight per thread
 
+template <int TOPL>
 __device__ __forceinline__ void list_insert(unsigned long long (&Lst)[TOPL], unsigned long long o) {
-    if (o > Lst[TOPL - 1]) {
-        Lst[TOPL - 1] = o;
+    Lst[TOPL - 1] = o;
 #pragma unroll
-        for (int i = TOPL - 1; i > 0; --i) {
-            if (Lst[i] > Lst[i - 1]) {
-                unsigned long long t = Lst[i];
-                Lst[i] = Lst[i - 1];
-                Lst[i - 1] = t;
-            }
+    for (int i = TOPL - 1; i > 0; --i) {
+        if (Lst[i] > Lst[i - 1]) {
+            const unsigned long long t = Lst[i];
+            Lst[i] = Lst[i - 1];
+            Lst[i - 1] = t;
         }
     }
 }
 
-template <bool VEC>
-__global__ void __launch_bounds__(NT) k_cache_build(CacheArgs a) {
-    __shared__ unsigned long long redu[NWARP];
+// TOPL: per-thread list length (4 when every fan-out is at most 4, else 8)
+template <bool VEC, int TOPL>
+__global__ void __launch_bounds__(NTC, 4) k_cache_build(CacheArgs a) {
+    __shared__ unsigned long long redu[NTC / 32];
     const int row = blockIdx.x, tid = threadIdx.x;
     const int b = row / a.K, d = row % a.K;
     const int Fd = a.F[d];
@@ -50,36 +53,51 @@ __global__ void __launch_bounds__(NT) k_cache_build(CacheArgs a) {
             unsigned long long Lst[TOPL];
 #pragma unroll
             for (int i = 0; i < TOPL; ++i) Lst[i] = 0ull;
-            // an element can only enter the list when its raw bits reach those
-            // of the current 8th best (positive floats order like their bits;
-            // negative or NaN q pass this test and are rejected below)
-            uint32_t thr = (uint32_t)(Lst[TOPL - 1] >> 32) & 0x7FFFFFFFu;
+            // An element can only enter the list when its raw bits reach thr,
+            // those of the list's last entry (at least 1: q > 0).  Positive
+            // floats order like their bits; negative or NaN q pass this test
+            // and are rejected below.
+            uint32_t thr = 1u;
             auto consider = [&](float qv, int x) {
-                if (__float_as_uint(qv) < thr) return;
                 if (!(qv > 0.0f) || x == xd) return;
                 const unsigned long long o = order_val(__float_as_uint(qv) | 0x80000000u, (uint32_t)x);
                 if (o < ub && o > Lst[TOPL - 1]) {
-                    list_insert(Lst, o);
-                    thr = (uint32_t)(Lst[TOPL - 1] >> 32) & 0x7FFFFFFFu;
+                    list_insert<TOPL>(Lst, o);
+                    const uint32_t t = (uint32_t)(Lst[TOPL - 1] >> 32) & 0x7FFFFFFFu;
+                    thr = t > 1u ? t : 1u;
                 }
             };
             if (VEC) {
                 const int nch = a.V >> 2;
-#pragma unroll 4
-                for (int cc = tid; cc < nch; cc += NT) {
-                    const uint4 w = ldg16(qr + (size_t)cc * 4);
-                    consider(__uint_as_float(w.x), cc * 4);
-                    consider(__uint_as_float(w.y), cc * 4 + 1);
-                    consider(__uint_as_float(w.z), cc * 4 + 2);
-                    consider(__uint_as_float(w.w), cc * 4 + 3);
+                for (int c0 = tid; c0 < nch; c0 += NTC * CLD) {
+                    uint4 w[CLD];
+#pragma unroll
+                    for (int u = 0; u < CLD; ++u) {
+                        const int cc = c0 + u * NTC;
+                        w[u] = cc < nch ? ldg16(qr + (size_t)cc * 4) : make_uint4(0u, 0u, 0u, 0u);
+                    }
+#pragma unroll
+                    for (int u = 0; u < CLD; ++u) {
+                        // one test per four values: the largest raw bits
+                        if (max(max(w[u].x, w[u].y), max(w[u].z, w[u].w)) >= thr) {
+                            const int x0 = (c0 + u * NTC) * 4;
+                            if (w[u].x >= thr) consider(__uint_as_float(w[u].x), x0);
+                            if (w[u].y >= thr) consider(__uint_as_float(w[u].y), x0 + 1);
+                            if (w[u].z >= thr) consider(__uint_as_float(w[u].z), x0 + 2);
+                            if (w[u].w >= thr) consider(__uint_as_float(w[u].w), x0 + 3);
+                        }
+                    }
                 }
             } else {
-                for (int x = tid; x < a.V; x += NT) consider(__ldg(qr + x), x);
+                for (int x = tid; x < a.V; x += NTC) {
+                    const float qv = __ldg(qr + x);
+                    if (__float_as_uint(qv) >= thr) consider(qv, x);
+                }
             }
             const int take = min(TOPL, Fd - got);
             bool exhausted = false;
             for (int t = 0; t < take; ++t) {
-                unsigned long long best = block_reduce(Lst[0], redu, MaxU64());
+                const unsigned long long best = block_reduce_n<NTC>(Lst[0], redu, MaxU64());
                 if (best == 0ull) {
                     exhausted = true;
                     break;
@@ -99,7 +117,7 @@ __global__ void __launch_bounds__(NT) k_cache_build(CacheArgs a) {
             if (exhausted) break;
         }
     }
-    for (int j = got + tid; j < Fd; j += NT) {
+    for (int j = got + tid; j < Fd; j += NTC) {
         bt[j] = -1;
         bp[j] = 0.0f;
     }
@@ -128,8 +146,16 @@ __global__ void k_cache_lookup(const int32_t *bt, CacheArgs a, const int32_t *ac
 }
 
 cudaError_t launch_cache_build(const CacheArgs &a, bool vec, cudaStream_t s) {
-    if (vec) k_cache_build<true><<<a.B * a.K, NT, 0, s>>>(a);
-    else k_cache_build<false><<<a.B * a.K, NT, 0, s>>>(a);
+    int fmax = 0;
+    for (int d = 0; d < a.K; ++d) fmax = a.F[d] > fmax ? a.F[d] : fmax;
+    const int g = a.B * a.K;
+    if (fmax <= 4) {
+        if (vec) k_cache_build<true, 4><<<g, NTC, 0, s>>>(a);
+        else k_cache_build<false, 4><<<g, NTC, 0, s>>>(a);
+    } else {
+        if (vec) k_cache_build<true, 8><<<g, NTC, 0, s>>>(a);
+        else k_cache_build<false, 8><<<g, NTC, 0, s>>>(a);
+    }
     return cudaGetLastError();
 }
 
