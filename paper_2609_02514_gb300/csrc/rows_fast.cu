@@ -32,6 +32,7 @@
 //            draft token at this position, per-row state for the resolve
 //            kernels.
 #include <climits>
+#include <type_traits>
 #include <cuda_bf16.h>
 
 #include "common.cuh"
@@ -166,6 +167,7 @@ __global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
     __shared__ uint32_t bins[NBIN];
     __shared__ float redf[NWF], redk[NWF], redh[NWF], redl[NWF];
     __shared__ int s_ncand, s_ngl, s_bc, s_nstar, s_L;
+    __shared__ uint32_t s_thr;
     __shared__ double s_S, s_Snuc;
     __shared__ float s_inv_S;
     __shared__ unsigned long long s_cut, s_Snuc_fx, s_cumL_fx;
@@ -189,7 +191,10 @@ __global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
     float t1 = -INFINITY, t2 = -INFINITY;  // this thread's two largest group maxima
     // groups per iteration: eight 16-byte loads in flight per thread
     constexpr int GPI = GC >= 8 ? 1 : 8 / GC;
-    for (int g0 = tid; g0 < ng; g0 += NTF * GPI) {
+    const int ngf = nch / GC;  // groups without a ragged end
+    // one iteration: GPI groups, one reference check and one compensated add
+    auto step = [&](int g0, auto checked) {
+        constexpr bool CHK = decltype(checked)::value;
         uint4 w[GPI][GC];
 #pragma unroll
         for (int h = 0; h < GPI; ++h) {
@@ -197,34 +202,45 @@ __global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
 #pragma unroll
             for (int j = 0; j < GC; ++j) {
                 const int cc = g * GC + j;
-                w[h][j] = (g < ng && cc < nch) ? ldg16(row + (size_t)cc * 16) : make_uint4(NI, NI, NI, NI);
+                w[h][j] = (!CHK || (g < ng && cc < nch)) ? ldg16(row + (size_t)cc * 16) : make_uint4(NI, NI, NI, NI);
             }
         }
+        float im = -INFINITY;
 #pragma unroll
         for (int h = 0; h < GPI; ++h) {
             const int g = g0 + h * NTF;
             const float gm = group_max<DT, GC>(w[h]);
-            m_t = fmaxf(m_t, gm);
+            im = fmaxf(im, gm);
             if (gm > t2) {
                 t2 = fminf(gm, t1);
                 t1 = fmaxf(gm, t1);
             }
-            const float gk = gm * a.c;
-            if (gk > k_t) {
-                const float nk = ceilf(gk);
-                const float sc = pow2_int(k_t - nk);
-                s_t *= sc;
-                e_t *= sc;
-                k_t = nk;
-            }
-            const float gs = group_expsum<DT, GC>(w[h], a.c, -k_t);
-            const float t = s_t + gs;
-            if (fabsf(s_t) >= fabsf(gs)) e_t += (s_t - t) + gs;
-            else e_t += (gs - t) + s_t;
-            s_t = t;
-            if (g < ng) sketch[g] = Sketch<DT>::enc(fkey(gm));
+            if (!CHK || g < ng) sketch[g] = Sketch<DT>::enc(fkey(gm));
         }
-    }
+        m_t = fmaxf(m_t, im);
+        const float gk = im * a.c;
+        if (gk > k_t) {
+            const float nk = ceilf(gk);
+            const float sc = pow2_int(k_t - nk);
+            s_t *= sc;
+            e_t *= sc;
+            k_t = nk;
+        }
+        float gs[GPI];
+#pragma unroll
+        for (int h = 0; h < GPI; ++h) gs[h] = group_expsum<DT, GC>(w[h], a.c, -k_t);
+#pragma unroll
+        for (int wdt = 1; wdt < GPI; wdt <<= 1)
+#pragma unroll
+            for (int h = 0; h < GPI; h += 2 * wdt) gs[h] += gs[h + wdt];
+        const float t = s_t + gs[0];
+        if (fabsf(s_t) >= fabsf(gs[0])) e_t += (s_t - t) + gs[0];
+        else e_t += (gs[0] - t) + s_t;
+        s_t = t;
+    };
+    int g0 = tid;
+    for (; g0 + (GPI - 1) * NTF < ngf; g0 += NTF * GPI) step(g0, std::false_type());
+    for (; g0 < ng; g0 += NTF * GPI) step(g0, std::true_type());
     // dependent loads of the accept test, consumed at the end
     float zx = 0.f, qx = 0.f;
     if (xb >= 0 && xb < a.V) {
@@ -334,8 +350,23 @@ __global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
             const unsigned bal = __ballot_sync(0xffffffffu, hit >= 0);
             const int first = bal ? __ffs(bal) - 1 : -1;
             const int bc = first >= 0 ? __shfl_sync(0xffffffffu, hit, first) : -1;
+            // Bins are monotone in the order key, so a binary search finds
+            // the smallest sketch key in a bin <= bc; the scans below then
+            // select exactly those ids by integer compares.
+            uint32_t thr = 0;
+            if (bc >= 0) {
+                const float lim = (float)(bc + 1);
+                uint32_t lo = 0, hi = Sketch<DT>::enc(fkey(m));  // the max itself is in bin 0
+                while (lo < hi) {
+                    const uint32_t mid = lo + ((hi - lo) >> 1);
+                    if ((m - Sketch<DT>::dec((SK)mid)) * a.inv_w < lim) hi = mid;
+                    else lo = mid + 1;
+                }
+                thr = hi;
+            }
             if (lane == 0) {
                 s_bc = bc;
+                s_thr = thr;
                 s_ncand = 0;
                 s_ngl = 0;
             }
@@ -352,49 +383,52 @@ __global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
         if (tid == 0) fallback_row(a, r);
         return;
     }
-    // ---- candidates: every id whose bin is <= bc.  Bins are monotone in the
-    // order key, so a binary search finds the smallest sketch key in a bin
-    // <= bc and the scans below select exactly those ids by integer compares.
-    const float lim = (float)(bc + 1);
-    uint32_t thr;
-    {
-        uint32_t lo = 0, hi = Sketch<DT>::enc(fkey(m));  // the max itself is in bin 0
-        while (lo < hi) {
-            const uint32_t mid = lo + ((hi - lo) >> 1);
-            if ((m - Sketch<DT>::dec((SK)mid)) * a.inv_w < lim) hi = mid;
-            else lo = mid + 1;
-        }
-        thr = hi;
-    }
+    // ---- candidates: every id whose key reaches thr (bin <= bc) ----
+    const uint32_t thr = s_thr;
     const uint32_t thr_key = DT == ACES_BF16 ? thr << 16 : thr;  // for 32-bit element keys
     // groups holding candidates: the sketch is scanned 16 bytes at a time
-    // with packed compares; hits are listed in cand[] (free until ranking)
+    // with packed compares; each warp lists its hits in cand[] (free until
+    // ranking) with one atomic per warp and round
     int *glist = reinterpret_cast<int *>(cand);
     {
         constexpr int SPW = 16 / sizeof(SK);  // sketch entries per 16-byte word
         const int nw = (ng + SPW - 1) / SPW;
         const uint4 *sk4 = reinterpret_cast<const uint4 *>(sketch);
-        for (int i = tid; i < nw; i += NTF) {
-            const uint4 wd = sk4[i];
-            const uint32_t x[4] = {wd.x, wd.y, wd.z, wd.w};
-            unsigned any = 0;
-            if (DT == ACES_BF16) {
-                const uint32_t t2x = thr * 0x00010001u;
+        for (int i0 = 0; i0 < nw; i0 += NTF) {  // warp-uniform rounds
+            const int i = i0 + tid;
+            unsigned hm = 0;  // hit mask over the word's SPW entries
+            if (i < nw) {
+                const uint4 wd = sk4[i];
+                const uint32_t x[4] = {wd.x, wd.y, wd.z, wd.w};
+                if (DT == ACES_BF16) {
+                    const uint32_t t2x = thr * 0x00010001u;
 #pragma unroll
-                for (int q = 0; q < 4; ++q) any |= __vcmpgeu2(x[q], t2x);
-            } else {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) any |= x[q] >= thr;
-            }
-            if (any) {
-#pragma unroll
-                for (int e = 0; e < SPW; ++e) {
-                    const int g = i * SPW + e;
-                    if (g < ng && (uint32_t)sketch[g] >= thr) {
-                        const int pos = atomicAdd(&s_ngl, 1);
-                        if (pos < CAND_CAP_F) glist[pos] = g;
+                    for (int q = 0; q < 4; ++q) {
+                        const uint32_t c = __vcmpgeu2(x[q], t2x);
+                        hm |= ((c >> 15) & 1u) << (2 * q) | ((c >> 31) & 1u) << (2 * q + 1);
                     }
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) hm |= (unsigned)(x[q] >= thr) << q;
                 }
+                if (i == nw - 1 && ng % SPW) hm &= (1u << (ng % SPW)) - 1u;  // past the last group
+            }
+            if (!__any_sync(0xffffffffu, hm != 0u)) continue;
+            const int cnt = __popc(hm);
+            int inc = cnt;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int t = __shfl_up_sync(0xffffffffu, inc, o);
+                if (lane >= o) inc += t;
+            }
+            int base = 0;
+            if (lane == 31) base = atomicAdd(&s_ngl, inc);
+            base = __shfl_sync(0xffffffffu, base, 31) + inc - cnt;
+            while (hm) {
+                const int e = __ffs(hm) - 1;
+                hm &= hm - 1u;
+                if (base < CAND_CAP_F) glist[base] = i * SPW + e;
+                ++base;
             }
         }
     }
@@ -445,6 +479,7 @@ __global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
         for (int i = tid; i < n; i += NTF) {
             const unsigned long long v = cv[i];
             int rank = 0;
+#pragma unroll 4
             for (int j = 0; j < n; ++j) rank += cv[j] > v;
             ord[rank] = v;
             efx[rank] = to_fx(ex2(fmaf(order_value(v), a.c, -kref)));
