@@ -261,8 +261,11 @@ def reference_arm(args, ws, rank):
 
 
 def config_of(w):
-    return {"workload": w.name if w.B == gen_B(w) else f"{w.name} (first {w.B} sequences)", "B": w.B, "K": w.K, "V": w.V, "logits": w.dtype, "T": w.T, "top_p": w.top_p,
-            "k": w.k, "F": list(w.F), "l2": "inputs (z 2.2 GB + q 4.2 GB) exceed the 129 MB L2; no flush",
+    zb = w.B * (w.K + 1) * w.V * (2 if w.dtype == "bf16" else 4)
+    qb = w.B * w.K * w.V * 4
+    return {"workload": w.name if w.B == gen_B(w) else f"{w.name} (first {w.B} sequences)", "B": w.B, "K": w.K,
+            "V": w.V, "logits": w.dtype, "T": w.T, "top_p": w.top_p, "k": w.k, "F": list(w.F),
+            "l2": f"inputs (z {zb / 1e9:.2f} GB + q {qb / 1e9:.2f} GB) exceed the 129 MB L2; no flush",
             "parallelism": "one process per GPU, sequences sharded, no collective"}
 
 
