@@ -297,7 +297,9 @@ constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual s
 
 // Workspace layout (all offsets 16-byte aligned)
 struct Workspace {
-    int *fb_count;             // [4]   [0] rows handed to the general path, [1] wait timeouts
+    int *fb_count;             // [4]   [0] rows handed to the general path, [1] wait timeouts,
+                               //       [2] rows certified by the full sketch, [3] rows ordered by
+                               //       bitonic sort (path counters, cleared by every call)
     RowStat *stats;            // [rows]
     int *acc;                  // [B*K] accept bits
     int *fb_list;              // [rows]

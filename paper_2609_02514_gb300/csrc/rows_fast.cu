@@ -298,6 +298,7 @@ __global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
         if (pass == 1) {  // second tier: every group of the sketch
             __syncthreads();
             if (s_bc >= 0) break;
+            if (tid == 0) atomicAdd(&a.ws.fb_count[2], 1);
             for (int i = tid; i < NBIN; i += NTF) bins[i] = 0u;
             __syncthreads();
             for (int g = tid; g < ng; g += NTF) {
@@ -485,6 +486,7 @@ __global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
             efx[rank] = to_fx(ex2(fmaf(order_value(v), a.c, -kref)));
         }
     } else {
+        if (tid == 0) atomicAdd(&a.ws.fb_count[3], 1);
         const int np = next_pow2(n);
         for (int i = tid; i < np; i += NTF) ord[i] = i < n ? cv[i] : 0ull;
         __syncthreads();

@@ -1,0 +1,106 @@
+"""Parity on inputs built to drive each branch of the fast row kernel.
+
+The workspace's first four int32 words count, per call, the rows handed to
+the exact general kernel, bounded-wait timeouts, rows certified only by the
+full sketch histogram (the per-thread top-two maxima were not enough), and
+rows whose candidates were ordered by bitonic sort (more than 512).  Each
+test asserts the branch it targets was taken, then compares every output
+with the float64 oracle under the rules of tests/parity.py.
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+
+import gen
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def A():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2609_02514_gb300 as A
+    A.load()
+    return A
+
+
+def _run(A, orc, w, z):
+    """Verify the generator's q, x~, u with the logits z on both sides."""
+    inp = gen.generate(w)
+    inp["z"] = z
+    if z.dtype == np.uint16:
+        zt = torch.from_numpy(z.view(np.int16)).cuda().view(torch.bfloat16)
+    else:
+        zt = torch.from_numpy(z).cuda()
+    q, xt, u = (torch.from_numpy(inp[key]).cuda() for key in ("q", "xt", "u"))
+    ws = torch.zeros(A.workspace_bytes(w.B, w.K, w.V, w.k), dtype=torch.uint8, device="cuda")
+    g = A.verify(zt, q, xt, u, w.T, w.top_p, w.k, workspace=ws)
+    torch.cuda.synchronize()
+    g = {key: v.cpu().numpy() for key, v in g.items()}
+    counters = ws[:16].view(torch.int32).cpu().numpy().tolist()
+    o = orc.verify(z, inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
+    res = parity.compare_verify(inp, g, o, w.top_p, z.dtype == np.uint16, w.k)
+    return counters, res
+
+
+def _plateau(B, K, V, n_hot, group, seed):
+    """-30 everywhere except n_hot ids, one per sketch group, near 0."""
+    rng = np.random.default_rng(seed)
+    z = np.full((B, K + 1, V), -30.0, np.float32)
+    j = np.arange(n_hot)
+    ids = j * group + (j % group)
+    for b in range(B):
+        for i in range(K + 1):
+            z[b, i, ids] = rng.uniform(0.0, 1.5, n_hot).astype(np.float32)
+    return z
+
+
+def test_second_tier_certification_and_bitonic_order(A, orc):
+    # 1500 near-equal ids in 1500 different groups of 8 float32 logits: the
+    # 512 per-thread top maxima carry too little mass, the full sketch
+    # certifies, and the nucleus (~1200 ids) is ordered by bitonic sort
+    w = gen.make_workload(2, 2, 32000, "f32", T=1.0, top_p=0.8, k=64, seed=31)
+    counters, res = _run(A, orc, w, _plateau(2, 2, 32000, 1500, 8, 31))
+    fallback, timeouts, second_tier, bitonic = counters
+    assert fallback == 0 and timeouts == 0
+    assert second_tier == 6 and bitonic == 6, counters
+    assert res["checked_seqs"] == 2
+
+
+def test_more_candidates_than_capacity_falls_back(A, orc):
+    # 3000 near-equal ids: the nucleus alone exceeds the 2048 candidates the
+    # fast kernel holds, so every row goes to the exact general kernel
+    w = gen.make_workload(2, 1, 32000, "f32", T=1.0, top_p=0.8, k=32, seed=32)
+    counters, res = _run(A, orc, w, _plateau(2, 1, 32000, 3000, 8, 32))
+    assert counters[0] == 4, counters
+    assert res["checked_seqs"] == 2
+
+
+def test_first_tier_suffices_on_the_benchmark_rows(A, orc):
+    # the first 4 sequences of the 256000-id benchmark workload (68 rows):
+    # nearly every row is certified by the per-thread top maxima, and all
+    # are ranked directly on the fast path
+    w = dataclasses.replace(gen.WORKLOADS["b256_k16_v256000_bf16"], B=4)
+    z = gen.generate(w)["z"]
+    counters, res = _run(A, orc, w, z)
+    fallback, timeouts, second_tier, bitonic = counters
+    assert fallback == 0 and timeouts == 0 and bitonic == 0, counters
+    assert second_tier <= 3, counters
+    assert res["checked_seqs"] >= 3
+
+
+@pytest.mark.parametrize("dtype,V", [("bf16", 600000), ("f32", 300000), ("f32", 600000)],
+                         ids=["bf16_gc8", "f32_gc8", "f32_general"])
+def test_large_vocabularies(A, orc, dtype, V):
+    # bf16 at 600000 ids and f32 at 300000 use 8 chunks per sketch group;
+    # f32 at 600000 exceeds the sketch and runs on the general kernel
+    w = gen.make_workload(1, 1, V, dtype, T=0.8, top_p=0.9, k=48, seed=34)
+    z = gen.generate(w)["z"]
+    counters, res = _run(A, orc, w, z)
+    assert counters[1] == 0
+    assert res["checked_seqs"] == 1
