@@ -34,6 +34,8 @@
  *                                                     (Sec. III-C, Alg. 1)
  *   8. lookup:    key w = (pi, token) -> slot, -1 miss, -2 full accept
  *                                                     (Sec. III-B, Alg. 1)
+ *   9. sparse resample on the edge from the payload of row pi alone
+ *                 (Alg. 1 RESAMPLE; see orc_resample_sparse)
  *
  * Sums use Neumaier compensation in float64; sorting uses the C library's
  * qsort as the sorting primitive.
@@ -406,6 +408,165 @@ int orc_cache_lookup(const int32_t *branch_tok, const int32_t *F, int B, int K,
             if (branch_tok[(size_t)b * total + off + j] == token[b]) { slot[b] = off + j; break; }
     }
     return 0;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Public: steps 1-2 alone: the nucleus-renormalised target p of `rows`    */
+/* rows (used to measure how far the sparse resample is from the exact    */
+/* residual).  p_out [rows, V]; row_status [rows].                          */
+int orc_warp(const float *z, int rows, int V, double T, double top_p, double *p_out,
+             int32_t *row_status) {
+    int err = 0;
+#pragma omp parallel
+    {
+        rowbuf rb;
+        int ok = rowbuf_init(&rb, V);
+        if (!ok) {
+#pragma omp atomic write
+            err = 1;
+        }
+#pragma omp for schedule(dynamic, 1)
+        for (int r = 0; r < rows; ++r) {
+            if (!ok) continue;
+            rowinfo ri = warp_row(z + (size_t)r * V, V, T, top_p, &rb);
+            row_status[r] = ri.status;
+            for (int x = 0; x < V; ++x) p_out[(size_t)r * V + x] = ri.status ? 0.0 : rb.p[x];
+        }
+        rowbuf_free(&rb);
+    }
+    return err;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Public: edge-side resample from the sparse payload (Alg. 1             */
+/* RESAMPLE(P^_target, Q); Sec. III-B: the cloud returns pi and the        */
+/* partial target distribution of row pi, the edge draws the token).       */
+/*                                                                         */
+/* The edge knows p only on the payload ids I (probs p^_I) and the mass    */
+/* tau = tail outside them.  Reading used here:                            */
+/*   pi < K:  p^(x) = p^_x on I; outside I the mass tau is spread like the */
+/*            draft, p^(x) = tau * q(x) / q_rest, q_rest = sum_{x not in I} */
+/*            q(x) (0 when q_rest = 0).  r^ = max(0, p^ - q), i.e.          */
+/*            max(0, p^_x - q(x)) on I and q(x) * max(0, tau/q_rest - 1)    */
+/*            outside.  When tau = 0 the draft row is read on I only.       */
+/*   pi = K:  the bonus draw uses the payload alone, r^ = p^_I.             */
+/*   Token: smallest id j with sum_{x <= j} r^(x) > u[b, K] * sum r^ (the   */
+/*   exact path's rule).  If sum r^ = 0 the draw uses p^_I.                 */
+/* When the nucleus of row pi fits in the payload, tau = 0 and p^ = p:     */
+/* the result is the exact residual draw.                                   */
+/*                                                                         */
+/* Inputs: accept_len [B]; the payload of every row, ids [B, K+1, k],       */
+/* probs [B, K+1, k] (float32), tail [B, K+1]; row_status [B, K+1] of the   */
+/* verification; q [B, K, V]; u [B, K+1].  Outputs: token [B] (-1 when row  */
+/* pi is NONFINITE, the payload is empty, or q is NaN/negative where it is  */
+/* read: status [B] gets ORC_ROW_NONFINITE / ORC_ROW_BAD_Q).                */
+/* Diagnostics (may be NULL): res_target, res_cj, res_cjm1, res_sum [B] as  */
+/* in orc_verify; dist [B, V] the normalised distribution drawn from.       */
+int orc_resample_sparse(const int32_t *accept_len, const int32_t *ids, const float *probs,
+                        const float *tail, const int32_t *row_status, const float *q,
+                        const float *u, int B, int K, int V, int k, int32_t *token,
+                        int32_t *status, double *res_target, double *res_cj, double *res_cjm1,
+                        double *res_sum, double *dist) {
+    int err = 0;
+#pragma omp parallel
+    {
+        double *r = (double *)malloc(sizeof(double) * (size_t)V);
+        char *in = (char *)malloc((size_t)V);
+        if (!r || !in) {
+#pragma omp atomic write
+            err = 1;
+        }
+#pragma omp for schedule(dynamic, 1)
+        for (int b = 0; b < B; ++b) {
+            if (!r || !in) continue;
+            const int R1 = K + 1;
+            const int pi = accept_len[b];
+            const size_t row = (size_t)b * R1 + (size_t)pi;
+            int32_t tok = -1;
+            int st = 0;
+            double tgt = NAN, cj = NAN, cjm1 = NAN, sr = NAN;
+            if (pi < 0 || pi > K || (row_status[row] & ORC_ROW_NONFINITE)) {
+                st = ORC_ROW_NONFINITE;
+            } else {
+                const int32_t *I = ids + row * (size_t)k;
+                const float *P = probs + row * (size_t)k;
+                const double tau = (double)tail[row];
+                for (int x = 0; x < V; ++x) { r[x] = 0.0; in[x] = 0; }
+                int n_in = 0;
+                for (int j = 0; j < k; ++j)
+                    if (I[j] >= 0 && I[j] < V) { in[I[j]] = 1; ++n_in; }
+                const float *qr = pi < K ? q + ((size_t)b * K + (size_t)pi) * (size_t)V : NULL;
+                int bad = 0;
+                if (qr) {
+                    /* payload ids: max(0, p^ - q) */
+                    for (int j = 0; j < k; ++j) {
+                        int32_t x = I[j];
+                        if (x < 0 || x >= V) continue;
+                        double qx = (double)qr[x];
+                        if (isnan(qx) || qx < 0.0) { bad = 1; break; }
+                        double d = (double)P[j] - qx;
+                        r[x] = d > 0.0 ? d : 0.0;
+                    }
+                    /* outside the payload: the tail spread like q */
+                    if (!bad && tau > 0.0) {
+                        nsum qs = {0, 0};
+                        for (int x = 0; x < V && !bad; ++x) {
+                            double qx = (double)qr[x];
+                            if (isnan(qx) || qx < 0.0) { bad = 1; break; }
+                            if (!in[x]) nadd(&qs, qx);
+                        }
+                        double q_rest = nval(&qs);
+                        double g = q_rest > 0.0 ? tau / q_rest - 1.0 : 0.0;
+                        if (!bad && g > 0.0)
+                            for (int x = 0; x < V; ++x)
+                                if (!in[x]) r[x] = (double)qr[x] * g;
+                    }
+                } else {
+                    for (int j = 0; j < k; ++j)
+                        if (I[j] >= 0 && I[j] < V) r[I[j]] = (double)P[j];
+                }
+                if (bad) {
+                    st = ORC_ROW_BAD_Q;
+                } else if (n_in > 0) {
+                    nsum s = {0, 0};
+                    for (int x = 0; x < V; ++x) nadd(&s, r[x]);
+                    sr = nval(&s);
+                    if (!(sr > 0.0)) { /* p^ <= q wherever it is known: draw from p^_I */
+                        for (int x = 0; x < V; ++x) r[x] = 0.0;
+                        for (int j = 0; j < k; ++j)
+                            if (I[j] >= 0 && I[j] < V) r[I[j]] = (double)P[j];
+                        nsum s2 = {0, 0};
+                        for (int x = 0; x < V; ++x) nadd(&s2, r[x]);
+                        sr = nval(&s2);
+                    }
+                    if (sr > 0.0) {
+                        tgt = (double)u[(size_t)b * R1 + K] * sr;
+                        nsum c = {0, 0};
+                        int last_pos = -1;
+                        for (int x = 0; x < V; ++x) {
+                            double before = nval(&c);
+                            nadd(&c, r[x]);
+                            if (r[x] > 0.0) last_pos = x;
+                            if (nval(&c) > tgt) { tok = x; cj = nval(&c); cjm1 = before; break; }
+                        }
+                        if (tok < 0) tok = last_pos;
+                    }
+                }
+            }
+            token[b] = tok;
+            if (status) status[b] = st;
+            if (res_target) res_target[b] = tgt;
+            if (res_cj) res_cj[b] = cj;
+            if (res_cjm1) res_cjm1[b] = cjm1;
+            if (res_sum) res_sum[b] = sr;
+            if (dist)
+                for (int x = 0; x < V; ++x)
+                    dist[(size_t)b * V + x] = (tok >= 0 && sr > 0.0) ? r[x] / sr : 0.0;
+        }
+        free(r);
+        free(in);
+    }
+    return err;
 }
 
 int orc_num_threads(void) {

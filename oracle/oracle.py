@@ -58,6 +58,8 @@ def _load():
             lib.orc_verify.argtypes = [P, P, P, P, I, I, I, D, D, I, P, P, P, P, P, P, P, P, P, P, P, P, P, P]
             lib.orc_cache_build.argtypes = [P, P, P, I, I, I, P, P]
             lib.orc_cache_lookup.argtypes = [P, P, I, I, P, P, P]
+            lib.orc_warp.argtypes = [P, I, I, D, D, P, P]
+            lib.orc_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P, P, P, P, P]
             lib.orc_num_threads.argtypes = []
             for f in (lib.orc_sparsify, lib.orc_verify, lib.orc_cache_build, lib.orc_cache_lookup,
                       lib.orc_num_threads):
@@ -183,3 +185,46 @@ def branch_alloc(B_alloc: int, gamma: int, alpha: float, beta: float):
     for kk in rema[:left]:
         ints[kk] += 1
     return real, ints
+
+
+def warp(z, T: float, top_p: float):
+    """Steps 1-2: the nucleus-renormalised target p of every row of z [..., V]."""
+    lib = _load()
+    zf = _logits_f32(z)
+    V = zf.shape[-1]
+    rows = zf.size // V
+    p = np.empty((rows, V), np.float64)
+    st = np.empty(rows, np.int32)
+    if lib.orc_warp(_ptr(zf), rows, V, float(T), float(top_p), _ptr(p), _ptr(st)):
+        raise MemoryError("oracle allocation failed")
+    return p.reshape(zf.shape), st.reshape(zf.shape[:-1])
+
+
+def resample_sparse(accept_len, ids, probs, tail, row_status, q, u):
+    """Step 9: the edge's draw from the payload of row pi (Alg. 1 RESAMPLE).
+
+    accept_len [B], ids/probs [B, K+1, k] (probs as float32), tail [B, K+1],
+    row_status [B, K+1], q [B, K, V], u [B, K+1].  Returns token, status,
+    the flag diagnostics and dist [B, V] (the normalised distribution drawn from).
+    """
+    lib = _load()
+    ids = np.ascontiguousarray(ids, np.int32)
+    B, R, k = ids.shape
+    K = R - 1
+    q = np.ascontiguousarray(q, np.float32)
+    V = q.shape[-1]
+    al = np.ascontiguousarray(accept_len, np.int32)
+    pr = np.ascontiguousarray(probs, np.float32)
+    tl = np.ascontiguousarray(tail, np.float32)
+    rs = np.ascontiguousarray(row_status, np.int32)
+    uu = np.ascontiguousarray(u, np.float32)
+    out = dict(token=np.empty(B, np.int32), status=np.empty(B, np.int32),
+               res_target=np.empty(B, np.float64), res_cj=np.empty(B, np.float64),
+               res_cjm1=np.empty(B, np.float64), res_sum=np.empty(B, np.float64),
+               dist=np.empty((B, V), np.float64))
+    o = out
+    if lib.orc_resample_sparse(_ptr(al), _ptr(ids), _ptr(pr), _ptr(tl), _ptr(rs), _ptr(q), _ptr(uu), B, K, V, k,
+                               _ptr(o["token"]), _ptr(o["status"]), _ptr(o["res_target"]), _ptr(o["res_cj"]),
+                               _ptr(o["res_cjm1"]), _ptr(o["res_sum"]), _ptr(o["dist"])):
+        raise MemoryError("oracle allocation failed")
+    return out

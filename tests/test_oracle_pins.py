@@ -342,3 +342,127 @@ def test_branch_allocation_golden(orc):
         a, b, c, d, rest = line.split(None, 4)
         _, ints = orc.branch_alloc(int(a), int(b), float(c), float(d))
         assert ints == [int(x) for x in rest.split()]
+
+
+# --------------------------------------------------------------------------
+# step 9: edge-side resample from the sparse payload (Alg. 1 RESAMPLE)
+
+
+def _sparse_case(ids0, probs0, tail0, q0, u_draw):
+    """One sequence, K = 1, rejected at position 0: payload of row 0 given."""
+    k = len(ids0)
+    ids = np.full((1, 2, k), -1, np.int32)
+    probs = np.zeros((1, 2, k), np.float32)
+    tail = np.ones((1, 2), np.float32)
+    ids[0, 0] = ids0
+    probs[0, 0] = probs0
+    tail[0, 0] = tail0
+    q = np.asarray([[q0]], np.float32)
+    u = np.array([[0.5, u_draw]], np.float32)
+    return dict(accept_len=np.array([0], np.int32), ids=ids, probs=probs, tail=tail,
+                row_status=np.zeros((1, 2), np.int32), q=q, u=u)
+
+
+@pytest.mark.parametrize("u_draw,token", [(0.5, 0), (0.9, 1)])
+def test_sparse_resample_tail_below_draft_mass(orc, u_draw, token):
+    # payload {0: 0.5, 1: 0.3}, tail 0.2; q uniform over 4 ids.  Outside the
+    # payload q holds 0.5 > 0.2, so the spread tail never exceeds q there:
+    # r^ = (0.25, 0.05, 0, 0).  u * 0.3 < 0.25 picks id 0, else id 1.
+    c = _sparse_case([0, 1], [0.5, 0.3], 0.2, [0.25, 0.25, 0.25, 0.25], u_draw)
+    o = orc.resample_sparse(c["accept_len"], c["ids"], c["probs"], c["tail"], c["row_status"], c["q"], c["u"])
+    assert o["token"][0] == token and o["status"][0] == 0
+    np.testing.assert_allclose(o["dist"][0], [0.25 / 0.3, 0.05 / 0.3, 0.0, 0.0], atol=1e-6)
+
+
+@pytest.mark.parametrize("u_draw,token", [(0.3, 1), (0.6, 2), (0.9, 3)])
+def test_sparse_resample_tail_spread_like_the_draft(orc, u_draw, token):
+    # q = (0.7, 0.2, 0.05, 0.05): outside the payload q holds 0.1 and the
+    # tail 0.2, so p^ = 2 q there and r^ = q = 0.05 on ids 2 and 3;
+    # on the payload r^ = (max(0, 0.5 - 0.7), 0.3 - 0.2) = (0, 0.1).
+    c = _sparse_case([0, 1], [0.5, 0.3], 0.2, [0.7, 0.2, 0.05, 0.05], u_draw)
+    o = orc.resample_sparse(c["accept_len"], c["ids"], c["probs"], c["tail"], c["row_status"], c["q"], c["u"])
+    assert o["token"][0] == token
+    np.testing.assert_allclose(o["dist"][0], [0.0, 0.5, 0.25, 0.25], atol=1e-6)
+    assert o["res_sum"][0] == pytest.approx(0.2, abs=1e-7)
+
+
+def test_sparse_resample_bonus_row_uses_the_payload(orc):
+    # pi = K: no draft row; the draw follows the payload probabilities
+    c = _sparse_case([3, 1, 2], [0.6, 0.3, 0.1], 0.0, [0.25] * 4, 0.95)
+    c["accept_len"][0] = 1
+    c["ids"][0, 1] = [3, 1, 2]
+    c["probs"][0, 1] = [0.6, 0.3, 0.1]
+    c["tail"][0, 1] = 0.0
+    o = orc.resample_sparse(c["accept_len"], c["ids"], c["probs"], c["tail"], c["row_status"], c["q"], c["u"])
+    np.testing.assert_allclose(o["dist"][0], [0.0, 0.3, 0.1, 0.6], atol=1e-7)
+    assert o["token"][0] == 3          # 0.95 > 0.3 + 0.1 in id order
+
+
+def test_sparse_resample_invalid_rows(orc):
+    c = _sparse_case([0, 1], [0.5, 0.3], 0.2, [-0.1, 0.5, 0.3, 0.3], 0.5)
+    o = orc.resample_sparse(c["accept_len"], c["ids"], c["probs"], c["tail"], c["row_status"], c["q"], c["u"])
+    assert o["token"][0] == -1 and o["status"][0] == orc.ROW_BAD_Q      # q < 0 on the payload
+    c = _sparse_case([0, 1], [0.5, 0.3], 0.2, [0.25] * 4, 0.5)
+    c["row_status"][0, 0] = orc.ROW_NONFINITE
+    o = orc.resample_sparse(c["accept_len"], c["ids"], c["probs"], c["tail"], c["row_status"], c["q"], c["u"])
+    assert o["token"][0] == -1 and o["status"][0] == orc.ROW_NONFINITE
+
+
+def _verify_then_resample(orc, seed, k, top_p=0.9, T=1.0, V=2000, n=300):
+    rng = np.random.default_rng(seed)
+    zd = rng.normal(0.0, 2.0, (n, 2, V))
+    z = (0.8 * zd + 0.6 * rng.normal(0.0, 2.0, (n, 2, V))).astype(np.float32)
+    qw = np.exp((zd[:, :1] - zd[:, :1].max(-1, keepdims=True)) / T)
+    q = (qw / qw.sum(-1, keepdims=True)).astype(np.float32)
+    xt = np.array([[np.searchsorted(np.cumsum(q[b, 0], dtype=np.float64), rng.random() * 0.999)] for b in range(n)],
+                  np.int32).clip(0, V - 1)
+    u = ((rng.integers(1, 1 << 24, size=(n, 2))) / float(1 << 24)).astype(np.float32)
+    ov = orc.verify(z, q, xt, u, T, top_p, k)
+    os_ = orc.resample_sparse(ov["accept_len"], ov["topk_ids"], ov["topk_probs"].astype(np.float32),
+                              ov["tail"].astype(np.float32), ov["row_status"], q, u)
+    p, _ = orc.warp(z, T, top_p)
+    return z, q, u, ov, os_, p
+
+
+def test_sparse_resample_is_the_exact_draw_when_the_nucleus_fits(orc):
+    # k >= every nucleus size: tail = 0 and p^ = p, so the edge's draw is the
+    # cloud's exact residual draw, token for token
+    z, q, u, ov, os_, p = _verify_then_resample(orc, 71, k=256, top_p=0.8, T=0.5)
+    assert ov["n_nuc"].max() <= 256
+    n = len(u)
+    pi = ov["accept_len"]
+    same = 0
+    for b in range(n):
+        s = ov["res_sum"][b]
+        t = ov["res_target"][b]
+        if any(np.isfinite(c) and abs(t - c) < 1e-6 * s for c in (ov["res_cj"][b], ov["res_cjm1"][b])):
+            continue
+        assert os_["token"][b] == ov["out_token"][b], b
+        same += 1
+        # the distribution drawn from is norm(max(0, p_pi - q_pi)) (or p_K)
+        r = p[b, pi[b]] - (q[b, 0] if pi[b] < 1 else 0.0)
+        r = np.maximum(r, 0.0)
+        if r.sum() == 0.0:
+            r = p[b, pi[b]]
+        np.testing.assert_allclose(os_["dist"][b], r / r.sum(), atol=1e-6)
+    assert same >= n - 3
+
+
+def test_sparse_resample_distance_shrinks_with_payload_size(orc):
+    # total-variation distance between the edge's distribution and the exact
+    # residual, averaged over sequences: 0 once k covers every nucleus, and
+    # never larger for a larger payload on these rows
+    tvs = []
+    for k in (4, 16, 64, 256):
+        z, q, u, ov, os_, p = _verify_then_resample(orc, 72, k=k, top_p=0.8, T=0.5, n=120)
+        pi = ov["accept_len"]
+        d = []
+        for b in range(len(u)):
+            r = np.maximum(p[b, pi[b]] - (q[b, 0] if pi[b] < 1 else 0.0), 0.0)
+            if r.sum() == 0.0:
+                r = p[b, pi[b]]
+            d.append(0.5 * np.abs(os_["dist"][b] - r / r.sum()).sum())
+        tvs.append(float(np.mean(d)))
+    assert tvs[0] > 0.01
+    assert all(a >= b - 1e-9 for a, b in zip(tvs, tvs[1:])), tvs
+    assert tvs[-1] < 1e-6, tvs
