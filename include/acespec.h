@@ -204,6 +204,39 @@ aces_status aces_cache_lookup(const int32_t *branch_tok, const int32_t *F_host, 
                               const int32_t *accept_len, const int32_t *token, int32_t *slot,
                               aces_stream_t stream);
 
+/*
+ * Edge-side resample from the sparse downlink payload (Alg. 1
+ * RESAMPLE(P^_target, Q); Sec. III-B): the edge receives pi and the payload
+ * of row pi and draws the corrected (pi < K) or bonus (pi = K) token itself,
+ * with its own draft row q_pi.
+ *
+ * The target p is known only on the payload ids I (probs p^_I) plus the
+ * mass tau = tail_mass outside them.  For pi < K the tail is spread like
+ * the draft, p^(x) = tau * q(x) / q_rest outside I (q_rest = draft mass
+ * outside I), and the token is drawn from norm(max(0, p^ - q)) with the
+ * rule of aces_verify (smallest id j whose prefix sum over ids 0..j
+ * exceeds u[b, K] times the total); if that is all zero, from p^_I.  For
+ * pi = K the token is drawn from p^_I.  When the nucleus of row pi has at
+ * most k ids, tau = 0 and the token equals aces_verify's out_token.
+ *
+ *   accept_len  [B]          int32 pi_b from aces_verify
+ *   topk_ids    [B, K+1, k]  int32, topk_probs [B, K+1, k] float32,
+ *   tail_mass   [B, K+1]     float32, row_status [B, K+1]: aces_verify's
+ *                            payload and status (only row pi_b is read)
+ *   draft_probs [B, K, V]    float32; row pi_b is read on the payload ids,
+ *                            and entirely when its tail_mass > 0
+ *   uniforms    [B, K+1]     float32; u[b, K] is the draw
+ * Outputs: token [B] int32 (-1 when row pi is NONFINITE, the payload is
+ *   empty, or q is NaN/negative where it is read); status [B] int32
+ *   (ACES_ROW_NONFINITE / ACES_ROW_BAD_Q for those cases, else 0).
+ * Limits: 1 <= B, 1 <= K <= ACES_MAX_K, 2 <= V <= ACES_MAX_V,
+ *   1 <= k <= min(V, ACES_MAX_TOPK).
+ */
+aces_status aces_resample_sparse(const int32_t *accept_len, const int32_t *topk_ids, const float *topk_probs,
+                                 const float *tail_mass, const int32_t *row_status, const float *draft_probs,
+                                 const float *uniforms, int B, int K, int V, int k, int32_t *token,
+                                 int32_t *status, aces_stream_t stream);
+
 /* Static English text for a status code. */
 const char *aces_status_string(aces_status s);
 

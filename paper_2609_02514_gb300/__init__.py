@@ -62,9 +62,11 @@ def load():
         lib.aces_sparsify.argtypes = [P, I, I, I, F, F, I, P, P, P, P, P, S, P]
         lib.aces_cache_build.argtypes = [P, P, P, I, I, I, P, P, P]
         lib.aces_cache_lookup.argtypes = [P, P, I, I, P, P, P, P]
+        lib.aces_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P]
         lib.aces_status_string.argtypes = [I]
         lib.aces_status_string.restype = ctypes.c_char_p
-        for f in (lib.aces_verify, lib.aces_sparsify, lib.aces_cache_build, lib.aces_cache_lookup):
+        for f in (lib.aces_verify, lib.aces_sparsify, lib.aces_cache_build, lib.aces_cache_lookup,
+                  lib.aces_resample_sparse):
             f.restype = I
         _lib = lib
         return lib
@@ -209,3 +211,31 @@ def cache_lookup(branch_tok, F, accept_len, token, out: torch.Tensor | None = No
     code = lib.aces_cache_lookup(_p(bt), _f_host(F), B, K, _p(al), _p(tk), _p(slot), _stream(al.device))
     _check("aces_cache_lookup", code)
     return slot
+
+
+def resample_sparse(accept_len, topk_ids, topk_probs, tail_mass, row_status, draft_probs, uniforms,
+                    out: dict | None = None):
+    """Edge-side draw from the sparse payload of row pi (Alg. 1 RESAMPLE).
+
+    accept_len [B], topk_ids / topk_probs [B,K+1,k], tail_mass / row_status
+    [B,K+1] (as written by verify), draft_probs [B,K,V] float32, uniforms
+    [B,K+1] float32 -> token [B] int32, status [B] int32.
+    """
+    lib = load()
+    al = _cuda(accept_len, "accept_len")
+    ids = _cuda(topk_ids, "topk_ids")
+    pr = _cuda(topk_probs, "topk_probs")
+    tl = _cuda(tail_mass, "tail_mass")
+    st = _cuda(row_status, "row_status")
+    q = _cuda(draft_probs, "draft_probs")
+    u = _cuda(uniforms, "uniforms")
+    B, K, V = q.shape
+    k = ids.shape[-1]
+    dev = q.device
+    o = {} if out is None else dict(out)
+    o.setdefault("token", torch.empty(B, dtype=torch.int32, device=dev))
+    o.setdefault("status", torch.empty(B, dtype=torch.int32, device=dev))
+    code = lib.aces_resample_sparse(_p(al), _p(ids), _p(pr), _p(tl), _p(st), _p(q), _p(u), B, K, V, k,
+                                    _p(o["token"]), _p(o["status"]), _stream(dev))
+    _check("aces_resample_sparse", code)
+    return o

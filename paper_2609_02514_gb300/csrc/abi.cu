@@ -247,6 +247,24 @@ aces_status aces_cache_lookup(const int32_t *branch_tok, const int32_t *F_host, 
     return ACES_OK;
 }
 
+aces_status aces_resample_sparse(const int32_t *accept_len, const int32_t *topk_ids, const float *topk_probs,
+                                 const float *tail_mass, const int32_t *row_status, const float *draft_probs,
+                                 const float *uniforms, int B, int K, int V, int k, int32_t *token,
+                                 int32_t *status, aces_stream_t stream) {
+    if (B < 1 || K < 1 || K > ACES_MAX_K || V < 2 || V > ACES_MAX_V) return ACES_ERR_INVALID_ARG;
+    if (k < 1 || k > ACES_MAX_TOPK || k > V) return ACES_ERR_INVALID_ARG;
+    if ((long long)B * (K + 1) > INT_MAX / 2) return ACES_ERR_INVALID_ARG;
+    if (!accept_len || !topk_ids || !topk_probs || !tail_mass || !row_status || !draft_probs || !uniforms ||
+        !token || !status)
+        return ACES_ERR_INVALID_ARG;
+    const bool vec = aligned16(draft_probs) && V % 4 == 0;
+    if (launch_resample_sparse(accept_len, topk_ids, topk_probs, tail_mass, row_status, draft_probs, uniforms, B,
+                               K, V, k, token, status, vec, reinterpret_cast<cudaStream_t>(stream)) !=
+        cudaSuccess)
+        return ACES_ERR_CUDA;
+    return ACES_OK;
+}
+
 const char *aces_status_string(aces_status s) {
     switch (s) {
         case ACES_OK: return "ok";

@@ -228,6 +228,23 @@ __device__ __forceinline__ unsigned long long to_fx(float x) {
     return sh >= 0 ? (mant << sh) : (sh > -64 ? (mant >> (-sh)) : 0ull);
 }
 
+// floor(u * R) exactly for a uniform u = M / 2^sh with a 24-bit integer M
+// (0 < u < 1), via a 128-bit product; clamped to R - 1
+__device__ __forceinline__ unsigned long long floor_u_times(float uu, unsigned long long R) {
+    int ex;
+    const float fr = frexpf(uu, &ex);
+    const unsigned long long M = (unsigned long long)ldexpf(fr, 24);
+    const int sh = 24 - ex;
+    const unsigned long long lo = M * R, hi = __umul64hi(M, R);
+    unsigned long long thr;
+    if (!(uu > 0.0f) || sh >= 128) thr = 0ull;
+    else if (sh >= 64) thr = hi >> (sh - 64);
+    else if (sh == 0) thr = lo;
+    else thr = (lo >> sh) | (hi << (64 - sh));
+    if (thr >= R) thr = R - 1ull;
+    return thr;
+}
+
 // ---------------------------------------------------------------------------
 // mbarrier and bulk async copy (global -> shared), CTA scope
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -433,6 +450,10 @@ aces_status verify_impl(const void *target_logits, aces_dtype dt, const float *d
                         int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
                         aces_stream_t stream);
 cudaError_t launch_cache_build(const CacheArgs &a, bool vec, cudaStream_t s);
+cudaError_t launch_resample_sparse(const int32_t *accept_len, const int32_t *ids, const float *probs,
+                                   const float *tail, const int32_t *row_status, const float *q,
+                                   const float *u, int B, int K, int V, int k, int32_t *token,
+                                   int32_t *status, bool vec, cudaStream_t s);
 cudaError_t launch_cache_lookup(const int32_t *bt, const CacheArgs &a, const int32_t *accept_len,
                                 const int32_t *token, int32_t *slot, cudaStream_t s);
 

@@ -81,22 +81,6 @@ __device__ __forceinline__ void mass_fx(const char *zrow, const float *qrow, int
     }
 }
 
-// floor(u * R) exactly, u = M / 2^sh with a 24-bit integer M (0 < u < 1)
-__device__ __forceinline__ unsigned long long floor_u_times(float uu, unsigned long long R) {
-    int ex;
-    const float fr = frexpf(uu, &ex);
-    const unsigned long long M = (unsigned long long)ldexpf(fr, 24);
-    const int sh = 24 - ex;
-    const unsigned long long lo = M * R, hi = __umul64hi(M, R);
-    unsigned long long thr;
-    if (!(uu > 0.0f) || sh >= 128) thr = 0ull;
-    else if (sh >= 64) thr = hi >> (sh - 64);
-    else if (sh == 0) thr = lo;
-    else thr = (lo >> sh) | (hi << (64 - sh));
-    if (thr >= R) thr = R - 1ull;
-    return thr;
-}
-
 __device__ __forceinline__ int first_reject(const Workspace &ws, int b, int K) {
     int pi = K;
     for (int i = 0; i < K; ++i)

@@ -101,3 +101,20 @@ def test_binding_refuses_host_tensors():
     z = torch.zeros(1, 3, 16)
     with pytest.raises(ValueError):
         A.verify(z, torch.zeros(1, 2, 16), torch.zeros(1, 2, dtype=torch.int32), torch.zeros(1, 3), 1.0, 0.9, 4)
+
+
+def _resample(lib, **kw):
+    a = dict(al=FAKE, ids=FAKE, probs=FAKE, tail=FAKE, st=FAKE, q=FAKE, u=FAKE, B=2, K=4, V=1000, k=8,
+             tok=FAKE, stat=FAKE, s=None)
+    a.update(kw)
+    return lib.aces_resample_sparse(a["al"], a["ids"], a["probs"], a["tail"], a["st"], a["q"], a["u"], a["B"],
+                                    a["K"], a["V"], a["k"], a["tok"], a["stat"], a["s"])
+
+
+@pytest.mark.parametrize("kw", [
+    dict(B=0), dict(K=0), dict(K=17), dict(V=1), dict(V=(1 << 20) + 1), dict(k=0), dict(k=257),
+    dict(V=10, k=11), dict(al=None), dict(ids=None), dict(probs=None), dict(tail=None), dict(st=None),
+    dict(q=None), dict(u=None), dict(tok=None), dict(stat=None),
+])
+def test_resample_sparse_rejects_invalid_arguments(lib, kw):
+    assert _resample(lib, **kw) == 1
