@@ -198,6 +198,14 @@ def resid_q_count(out, K, k):
     return int((ids[rej, al[rej]] >= 0).sum())
 
 
+def resample_bytes(B, K, V, k, n_spread):
+    """Algorithmic bytes of one aces_resample_sparse call: per sequence the
+    payload of row pi (ids, probs, tail, status), q at its ids, the length
+    and the uniform, the token and status; the whole q row pi for the
+    n_spread sequences whose payload has a positive tail."""
+    return B * (k * 12 + 4 + 4 + 4 + 4 + 8) + n_spread * V * 4
+
+
 def cache_bytes(B, K, V, S):
     return B * K * V * 4 + B * K * 4 + B * S * 8
 
@@ -409,6 +417,27 @@ def main():
                         "gbs": cb / (part_ms["cache_build"] * 1e-3) / 1e9, "kernels": ["k_cache_build"]},
         "cache_lookup": {"ms": part_ms["cache_lookup"], "kernels": ["k_cache_lookup"]},
     }
+    # edge-side draw from the sparse payload (Alg. 1 RESAMPLE), timed apart from the step
+    rs_out = A.resample_sparse(out["accept_len"], out["topk_ids"], out["topk_probs"], out["tail_mass"],
+                               out["row_status"], d["q"], d["u"])
+    for _ in range(3):
+        A.resample_sparse(out["accept_len"], out["topk_ids"], out["topk_probs"], out["tail_mass"],
+                          out["row_status"], d["q"], d["u"], out=rs_out)
+    r0 = torch.cuda.Event(enable_timing=True)
+    r1 = torch.cuda.Event(enable_timing=True)
+    r0.record(stream)
+    for _ in range(args.steps):
+        A.resample_sparse(out["accept_len"], out["topk_ids"], out["topk_probs"], out["tail_mass"],
+                          out["row_status"], d["q"], d["u"], out=rs_out)
+    r1.record(stream)
+    torch.cuda.synchronize()
+    rs_ms = r0.elapsed_time(r1) / args.steps
+    tail_pi = out["tail_mass"][torch.arange(B, device=dev), out["accept_len"].long()].cpu().numpy()
+    n_spread = int((tail_pi > 0).sum())
+    rb = resample_bytes(B, K, V, k, n_spread)
+    parts["resample_sparse"] = {"ms": rs_ms, "alg_bytes": rb, "gbs": rb / (rs_ms * 1e-3) / 1e9,
+                                "sequences_reading_whole_q_row": n_spread, "kernels": ["k_resample_sparse"],
+                                "note": "edge-side draw from row pi's payload; not part of the step"}
     for p in parts.values():
         if "gbs" in p:
             p["frac_of_peak"] = p["gbs"] / peak

@@ -16,7 +16,7 @@
 //      weights (p^ - q on I) are gathered;
 //   2. only when tau > 0: one pass over q_pi gives q_rest (compensated fp32)
 //      and, once the spread factor is known, a second pass gives the weight
-//      of every 2048-id tile;
+//      of every 2048-id tile (four tiles' loads in flight per thread);
 //   3. the draw: smallest id j whose prefix sum exceeds floor(u * R), with
 //      every weight an integer in units of 2^-52 (exact, order independent).
 #include "common.cuh"
@@ -28,6 +28,7 @@ constexpr int SEPT = 8;                // consecutive ids per thread
 constexpr int STILE = NTS * SEPT;      // ids per tile
 constexpr int SPAY = ACES_MAX_TOPK;    // payload entries
 constexpr int STILES = (ACES_MAX_V + STILE - 1) / STILE;
+constexpr int TPI = 4;                 // tiles per round of the q passes
 
 // floor(x * 2^52) of a float x in [0, 2^11) from its bits (0 for x <= 0 or NaN)
 __device__ __forceinline__ unsigned long long to_fx52(float x) {
@@ -80,6 +81,7 @@ __global__ void __launch_bounds__(NTS) k_resample_sparse(SparseArgs a) {
     __shared__ unsigned long long sw[SPAY];    // their weights (2^-52 units)
     __shared__ unsigned long long tsum[STILES];
     __shared__ unsigned long long red[NTS / 32];
+    __shared__ unsigned long long red4[TPI][NTS / 32];
     __shared__ float redh[NTS / 32], redl[NTS / 32];
     __shared__ int s_n, s_bad, s_tok, s_tile;
     __shared__ float s_gam;
@@ -146,26 +148,36 @@ __global__ void __launch_bounds__(NTS) k_resample_sparse(SparseArgs a) {
     }
 
     // ---- 2. the tail, spread like the draft (pi < K, tau > 0) ----
-    const int ntile = (V + STILE - 1) / STILE;
+    const int ntile = (V + STILE - 1) / STILE;  // 2048-id tiles
     bool spread = false;
     if (qr && tau > 0.0f) {
         float hi = 0.0f, lo = 0.0f;  // compensated sum of q outside the payload
         int bad = 0;
-        for (int x0 = tid * SEPT; x0 < V; x0 += STILE) {
-            float qv[SEPT];
-            load_q<VEC>(qr, V, x0, qv);
-            int j = lower_bound_id(sid, n, x0);
+        for (int t0 = 0; t0 < ntile; t0 += TPI) {  // TPI tiles' loads in flight
+            float qv[TPI][SEPT];
 #pragma unroll
-            for (int e = 0; e < SEPT; ++e) {
-                const int x = x0 + e;
-                if (x >= V) break;
-                if (!(qv[e] >= 0.0f)) bad = 1;
-                while (j < n && sid[j] < x) ++j;
-                if (j < n && sid[j] == x) continue;
-                const float t = hi + qv[e];
-                if (fabsf(hi) >= fabsf(qv[e])) lo += (hi - t) + qv[e];
-                else lo += (qv[e] - t) + hi;
-                hi = t;
+            for (int h = 0; h < TPI; ++h) {
+                const int x0 = (t0 + h) * STILE + tid * SEPT;
+                if (x0 < V) load_q<VEC>(qr, V, x0, qv[h]);
+            }
+#pragma unroll
+            for (int h = 0; h < TPI; ++h) {
+                const int x0 = (t0 + h) * STILE + tid * SEPT;
+                if (x0 >= V) break;
+                int j = lower_bound_id(sid, n, x0);
+#pragma unroll
+                for (int e = 0; e < SEPT; ++e) {
+                    const int x = x0 + e;
+                    if (x >= V) break;
+                    const float qx = qv[h][e];
+                    if (!(qx >= 0.0f)) bad = 1;
+                    while (j < n && sid[j] < x) ++j;
+                    if (j < n && sid[j] == x) continue;
+                    const float t = hi + qx;
+                    if (fabsf(hi) >= fabsf(qx)) lo += (hi - t) + qx;
+                    else lo += (qx - t) + hi;
+                    hi = t;
+                }
             }
         }
         if (bad) s_bad = 1;
@@ -204,26 +216,43 @@ __global__ void __launch_bounds__(NTS) k_resample_sparse(SparseArgs a) {
         const float gam = s_gam;
         for (int t = tid; t < ntile; t += NTS) tsum[t] = 0ull;
         __syncthreads();
-        // weight of every tile: q * gam outside the payload, sw on it
-        for (int t = 0; t < ntile; ++t) {
-            const int x0 = t * STILE + tid * SEPT;
-            unsigned long long loc = 0ull;
-            if (x0 < V) {
-                float qv[SEPT];
-                load_q<VEC>(qr, V, x0, qv);
+        // weight of every tile: q * gam outside the payload, sw on it;
+        // TPI tiles per round, one block reduction of TPI sums
+        for (int t0 = 0; t0 < ntile; t0 += TPI) {
+            float qv[TPI][SEPT];
+#pragma unroll
+            for (int h = 0; h < TPI; ++h) {
+                const int x0 = (t0 + h) * STILE + tid * SEPT;
+                if (x0 < V) load_q<VEC>(qr, V, x0, qv[h]);
+            }
+            unsigned long long loc[TPI];
+#pragma unroll
+            for (int h = 0; h < TPI; ++h) {
+                const int x0 = (t0 + h) * STILE + tid * SEPT;
+                loc[h] = 0ull;
+                if (x0 >= V) continue;
                 int j = lower_bound_id(sid, n, x0);
 #pragma unroll
                 for (int e = 0; e < SEPT; ++e) {
                     const int x = x0 + e;
                     if (x >= V) break;
                     while (j < n && sid[j] < x) ++j;
-                    loc += (j < n && sid[j] == x) ? sw[j] : to_fx52(qv[e] * gam);
+                    loc[h] += (j < n && sid[j] == x) ? sw[j] : to_fx52(qv[h][e] * gam);
                 }
             }
-            const unsigned long long ts = block_reduce_n<NTS>(loc, red, SumU64());
-            if (tid == 0) tsum[t] = ts;
+#pragma unroll
+            for (int h = 0; h < TPI; ++h) loc[h] = warp_sum(loc[h]);
+            if (lane == 0)
+#pragma unroll
+                for (int h = 0; h < TPI; ++h) red4[h][wid] = loc[h];
+            __syncthreads();
+            if (tid < TPI && t0 + tid < ntile) {
+                unsigned long long ts = 0ull;
+                for (int i = 0; i < NTS / 32; ++i) ts += red4[tid][i];
+                tsum[t0 + tid] = ts;
+            }
+            __syncthreads();
         }
-        __syncthreads();
         if (tid == 0) {
             unsigned long long tot = 0ull;
             for (int t = 0; t < ntile; ++t) tot += tsum[t];

@@ -466,3 +466,21 @@ def test_sparse_resample_distance_shrinks_with_payload_size(orc):
     assert tvs[0] > 0.01
     assert all(a >= b - 1e-9 for a, b in zip(tvs, tvs[1:])), tvs
     assert tvs[-1] < 1e-6, tvs
+
+
+def test_sparse_resample_tv_golden_table():
+    # the committed table of the edge's distance to the exact residual is
+    # reproduced by the oracle (two rows of the smallest workload)
+    import os
+    import sys
+    here = os.path.dirname(os.path.abspath(__file__))
+    sys.path.insert(0, os.path.join(here, "golden"))
+    import make_sparse_tv as mk
+    want = {}
+    for line in open(os.path.join(here, "golden", "sparse_resample_tv.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        f = line.split()
+        want[(f[0], int(f[1]))] = line.strip()
+    for k in (4, 64):
+        assert mk.fmt("b16_k8_v32000_f32", k, mk.row("b16_k8_v32000_f32", k)) == want[("b16_k8_v32000_f32", k)]
