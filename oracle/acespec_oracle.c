@@ -569,6 +569,76 @@ int orc_resample_sparse(const int32_t *accept_len, const int32_t *ids, const flo
     return err;
 }
 
+/* ---------------------------------------------------------------------- */
+/* Public: probability that the branch cache recovers the sequence (Sec.  */
+/* III-C, Eq. for P_hit): given the drafted chain x~ and the branches      */
+/* branch_tok [B, sum F], the only randomness left is the uniforms.  With  */
+/* a_i = min(1, p_i(x~_i) / q_i(x~_i)) (0 when q_i(x~_i) <= 0) and R_i the */
+/* mass of norm(max(0, p_i - q_i)) (of p_i when that is all zero) on the   */
+/* branches of depth i:                                                    */
+/*   hit_prob[b]   = sum_{i<K} (prod_{j<i} a_j)(1 - a_i) R_i + prod a_j    */
+/*                   (first rejection at i and its token cached, or the   */
+/*                   whole chain accepted: lookup slot >= 0 or -2);        */
+/*   paper_prob[b] = prod_{i<K} (a_i + (1 - a_i) R_i), the product form of */
+/*                   Sec. IV-C, evaluated with the same a_i and R_i.       */
+int orc_hit_prob(const float *z, const float *q, const int32_t *xt, int B, int K, int V, double T,
+                 double top_p, const int32_t *branch_tok, const int32_t *F, double *hit_prob,
+                 double *paper_prob) {
+    int err = 0;
+    int total = 0;
+    for (int d = 0; d < K; ++d) total += F[d];
+#pragma omp parallel
+    {
+        rowbuf rb;
+        int ok = rowbuf_init(&rb, V);
+        if (!ok) {
+#pragma omp atomic write
+            err = 1;
+        }
+#pragma omp for schedule(dynamic, 1)
+        for (int b = 0; b < B; ++b) {
+            if (!ok) continue;
+            double survive = 1.0, hit = 0.0, prod = 1.0;
+            int off = 0;
+            for (int i = 0; i < K; ++i) {
+                const float *zr = z + ((size_t)b * (K + 1) + i) * (size_t)V;
+                const float *qr = q + ((size_t)b * K + i) * (size_t)V;
+                rowinfo ri = warp_row(zr, V, T, top_p, &rb);
+                double a = 0.0, R = 0.0;
+                if (!ri.status) {
+                    int32_t x = xt[(size_t)b * K + i];
+                    if (x >= 0 && x < V && (double)qr[x] > 0.0) {
+                        double ratio = rb.p[x] / (double)qr[x];
+                        a = ratio < 1.0 ? ratio : 1.0;
+                    }
+                    nsum rs = {0, 0};
+                    for (int y = 0; y < V; ++y) {
+                        double d = rb.p[y] - (double)qr[y];
+                        nadd(&rs, d > 0.0 ? d : 0.0);
+                    }
+                    double Rt = nval(&rs);
+                    nsum cs = {0, 0};
+                    for (int j = 0; j < F[i]; ++j) {
+                        int32_t y = branch_tok[(size_t)b * total + off + j];
+                        if (y < 0 || y >= V) continue;
+                        double d = rb.p[y] - (double)qr[y];
+                        nadd(&cs, Rt > 0.0 ? (d > 0.0 ? d : 0.0) : rb.p[y]);
+                    }
+                    R = Rt > 0.0 ? nval(&cs) / Rt : nval(&cs);
+                }
+                hit += survive * (1.0 - a) * R;
+                survive *= a;
+                prod *= a + (1.0 - a) * R;
+                off += F[i];
+            }
+            hit_prob[b] = hit + survive;
+            if (paper_prob) paper_prob[b] = prod;
+        }
+        rowbuf_free(&rb);
+    }
+    return err;
+}
+
 int orc_num_threads(void) {
 #ifdef _OPENMP
     return omp_get_max_threads();

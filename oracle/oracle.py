@@ -59,6 +59,7 @@ def _load():
             lib.orc_cache_build.argtypes = [P, P, P, I, I, I, P, P]
             lib.orc_cache_lookup.argtypes = [P, P, I, I, P, P, P]
             lib.orc_warp.argtypes = [P, I, I, D, D, P, P]
+            lib.orc_hit_prob.argtypes = [P, P, P, I, I, I, D, D, P, P, P, P]
             lib.orc_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P, P, P, P, P]
             lib.orc_num_threads.argtypes = []
             for f in (lib.orc_sparsify, lib.orc_verify, lib.orc_cache_build, lib.orc_cache_lookup,
@@ -228,3 +229,23 @@ def resample_sparse(accept_len, ids, probs, tail, row_status, q, u):
                                _ptr(o["res_cjm1"]), _ptr(o["res_sum"]), _ptr(o["dist"])):
         raise MemoryError("oracle allocation failed")
     return out
+
+
+def hit_prob(z, q, xt, T: float, top_p: float, branch_tok, F):
+    """Per-sequence probability that the cache recovers the sequence (lookup
+    slot >= 0 or -2) given z, q, x~ and the branches, and the product form
+    prod_k (a_k + (1 - a_k) R_k) of Sec. IV-C with the same per-row terms."""
+    lib = _load()
+    zf = _logits_f32(z)
+    B, R, V = zf.shape
+    K = R - 1
+    q = np.ascontiguousarray(q, np.float32)
+    xt = np.ascontiguousarray(xt, np.int32)
+    bt = np.ascontiguousarray(branch_tok, np.int32)
+    Fa = np.ascontiguousarray(F, np.int32)
+    hp = np.empty(B, np.float64)
+    pp = np.empty(B, np.float64)
+    if lib.orc_hit_prob(_ptr(zf), _ptr(q), _ptr(xt), B, K, V, float(T), float(top_p), _ptr(bt), _ptr(Fa),
+                        _ptr(hp), _ptr(pp)):
+        raise MemoryError("oracle allocation failed")
+    return hp, pp

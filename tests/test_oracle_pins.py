@@ -484,3 +484,47 @@ def test_sparse_resample_tv_golden_table():
         want[(f[0], int(f[1]))] = line.strip()
     for k in (4, 64):
         assert mk.fmt("b16_k8_v32000_f32", k, mk.row("b16_k8_v32000_f32", k)) == want[("b16_k8_v32000_f32", k)]
+
+
+# --------------------------------------------------------------------------
+# cache hit probability (Sec. III-C; Eq. for P_hit in Sec. IV-C)
+
+
+def _hit_batch(orc, n, F, seed, V=16, K=3):
+    rng = np.random.default_rng(seed)
+    z_rows = rng.normal(0.0, 1.5, (K + 1, V))
+    q_rows = _softmax(z_rows[:K] + rng.normal(0.0, 1.0, (K, V)), 1.0).reshape(K, V)
+    z, q, xt, u = _batch(z_rows, q_rows, n, seed + 1)
+    return z, q, xt, u
+
+
+def test_hit_probability_matches_simulation_of_the_protocol(orc):
+    # the oracle's own verify + cache + lookup, repeated over uniforms, hits
+    # as often as the closed form predicts (5 sigma)
+    F = [3, 2, 1]
+    z, q, xt, u = _hit_batch(orc, 40000, F, 81)
+    ov = orc.verify(z, q, xt, u, 1.0, 1.0, 0)
+    bt, _ = orc.cache_build(q, xt, F)
+    slot = orc.cache_lookup(bt, F, ov["accept_len"], ov["out_token"])
+    hits = (slot >= 0) | (slot == -2)
+    hp, pp = orc.hit_prob(z, q, xt, 1.0, 1.0, bt, F)
+    sd = np.sqrt(np.sum(hp * (1 - hp))) / len(hp)
+    assert abs(hits.mean() - hp.mean()) < 5 * sd, (hits.mean(), hp.mean(), sd)
+    assert 0.2 < hp.mean() < 0.99
+
+
+def test_hit_probability_closed_forms(orc):
+    z, q, xt, u = _hit_batch(orc, 200, [0, 0, 0], 82)
+    ov = orc.verify(z, q, xt, u, 1.0, 1.0, 0)
+    a = np.minimum(1.0, ov["ratio"])
+    # no branches: only a fully accepted chain is recovered
+    bt0, _ = orc.cache_build(q, xt, [0, 0, 0])
+    hp, pp = orc.hit_prob(z, q, xt, 1.0, 1.0, bt0, [0, 0, 0])
+    np.testing.assert_allclose(hp, np.prod(a, axis=1), rtol=1e-12)
+    np.testing.assert_allclose(pp, np.prod(a, axis=1), rtol=1e-12)
+    # every alternative cached (q has full support here): always recovered
+    Fall = [15, 15, 15]
+    bt1, _ = orc.cache_build(q, xt, Fall)
+    hp, pp = orc.hit_prob(z, q, xt, 1.0, 1.0, bt1, Fall)
+    np.testing.assert_allclose(hp, 1.0, atol=1e-12)
+    np.testing.assert_allclose(pp, 1.0, atol=1e-12)
