@@ -237,6 +237,28 @@ aces_status aces_resample_sparse(const int32_t *accept_len, const int32_t *topk_
                                  const float *uniforms, int B, int K, int V, int k, int32_t *token,
                                  int32_t *status, aces_stream_t stream);
 
+/*
+ * Network-aware tree budget (Sec. IV-B, Eq. for B*(t)): the largest tree
+ * size B whose edge drafting time fits in the cloud turnaround,
+ * draft_latency_s[B - 1] <= rtt_s + verify_s, capped by B_max.  The host
+ * array draft_latency_s [n] is the measured tree-drafting time of sizes
+ * 1..n (non-decreasing; this tabulates the inverse latency function).
+ * *B_star = 0 when even one token does not fit.  The branch budget is then
+ * B_alloc = B* - gamma (Sec. IV-C).  Host-only; launches nothing.
+ */
+aces_status aces_tree_budget(const double *draft_latency_s, int n, double rtt_s, double verify_s, int B_max,
+                             int *B_star);
+
+/*
+ * Geometric-decay branch allocation (Sec. IV-C): with eta = alpha^(1/(beta+1)),
+ * F*_k = B_alloc (1 - eta) / (1 - eta^gamma) eta^k (uniform when eta = 1),
+ * rounded to integers summing to B_alloc: floor, then one more branch for
+ * each of the largest fractional parts, ties to the shallower depth.
+ * F_out [gamma] host int32.  0 < alpha <= 1, beta > 0, B_alloc >= 0,
+ * 1 <= gamma <= ACES_MAX_K.  Host-only; launches nothing.
+ */
+aces_status aces_branch_alloc(int B_alloc, int gamma, double alpha, double beta, int32_t *F_out);
+
 /* Static English text for a status code. */
 const char *aces_status_string(aces_status s);
 

@@ -63,10 +63,12 @@ def load():
         lib.aces_cache_build.argtypes = [P, P, P, I, I, I, P, P, P]
         lib.aces_cache_lookup.argtypes = [P, P, I, I, P, P, P, P]
         lib.aces_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P]
+        lib.aces_tree_budget.argtypes = [P, I, ctypes.c_double, ctypes.c_double, I, P]
+        lib.aces_branch_alloc.argtypes = [I, I, ctypes.c_double, ctypes.c_double, P]
         lib.aces_status_string.argtypes = [I]
         lib.aces_status_string.restype = ctypes.c_char_p
         for f in (lib.aces_verify, lib.aces_sparsify, lib.aces_cache_build, lib.aces_cache_lookup,
-                  lib.aces_resample_sparse):
+                  lib.aces_resample_sparse, lib.aces_tree_budget, lib.aces_branch_alloc):
             f.restype = I
         _lib = lib
         return lib
@@ -239,3 +241,22 @@ def resample_sparse(accept_len, topk_ids, topk_probs, tail_mass, row_status, dra
                                     _p(o["token"]), _p(o["status"]), _stream(dev))
     _check("aces_resample_sparse", code)
     return o
+
+
+def tree_budget(draft_latency_s, rtt_s: float, verify_s: float, B_max: int) -> int:
+    """Network-aware budget B* (Sec. IV-B) from the drafting times of tree sizes 1..n."""
+    lib = load()
+    n = len(draft_latency_s)
+    arr = (ctypes.c_double * n)(*[float(t) for t in draft_latency_s])
+    out = ctypes.c_int(0)
+    _check("aces_tree_budget", lib.aces_tree_budget(arr, n, float(rtt_s), float(verify_s), int(B_max),
+                                                    ctypes.byref(out)))
+    return int(out.value)
+
+
+def branch_alloc(B_alloc: int, gamma: int, alpha: float, beta: float) -> list:
+    """Integer branch counts F_0..F_{gamma-1} of the geometric-decay allocation (Sec. IV-C)."""
+    lib = load()
+    F = (ctypes.c_int32 * int(gamma))()
+    _check("aces_branch_alloc", lib.aces_branch_alloc(int(B_alloc), int(gamma), float(alpha), float(beta), F))
+    return [int(f) for f in F]
