@@ -528,3 +528,15 @@ def test_hit_probability_closed_forms(orc):
     hp, pp = orc.hit_prob(z, q, xt, 1.0, 1.0, bt1, Fall)
     np.testing.assert_allclose(hp, 1.0, atol=1e-12)
     np.testing.assert_allclose(pp, 1.0, atol=1e-12)
+
+
+def test_hit_rate_golden_table():
+    # the committed hit-rate table is reproduced by the oracle (one regime)
+    import os
+    import sys
+    here = os.path.dirname(os.path.abspath(__file__))
+    sys.path.insert(0, os.path.join(here, "golden"))
+    import make_hit_rates as mk
+    lines = [ln.strip() for ln in open(os.path.join(here, "golden", "hit_rates.txt")) if not ln.startswith("#")]
+    got = mk.rows(*mk.REGIMES[0])
+    assert got == lines[:len(got)]
