@@ -249,3 +249,43 @@ def hit_prob(z, q, xt, T: float, top_p: float, branch_tok, F):
                         _ptr(hp), _ptr(pp)):
         raise MemoryError("oracle allocation failed")
     return hp, pp
+
+
+def compact_kv(kv, prefix_len, accept_len, slot, K: int, branch_len: int):
+    """COMPACT_KV / ROLLBACK_KV of Alg. 1 on a KV array [planes, B, H, S, D].
+
+    The tree of every sequence is packed after its prefix of prefix_len[b]
+    positions: the main chain (K positions), then the branches in slot order,
+    branch_len positions each.  After the lookup:
+      slot >= 0  (hit):   the branch's rows move right behind the accepted
+                          tokens, positions t + pi ...; new length
+                          t + pi + branch_len;
+      slot == -2 (all accepted): nothing moves; new length t + K;
+      slot == -1 (miss):  the rejected drafts are dropped; new length t + pi.
+    A sequence whose tree would pass the end of the array gets new length -1
+    and nothing moves.  Returns (new kv, new lengths).  Plain slice copies.
+    """
+    kv = np.array(kv, copy=True)
+    S = kv.shape[3]
+    B = kv.shape[1]
+    new_len = np.empty(B, np.int32)
+    for b in range(B):
+        t, pi, s = int(prefix_len[b]), int(accept_len[b]), int(slot[b])
+        total = 0
+        if t < 0 or pi < 0 or pi > K:
+            new_len[b] = -1
+            continue
+        if s >= 0:
+            src = t + K + s * branch_len
+            if src + branch_len > S:
+                new_len[b] = -1
+                continue
+            block = kv[:, b, :, src:src + branch_len, :].copy()
+            kv[:, b, :, t + pi:t + pi + branch_len, :] = block
+            total = t + pi + branch_len
+        elif s == -2:
+            total = t + K
+        else:
+            total = t + pi
+        new_len[b] = total if total <= S else -1
+    return kv, new_len

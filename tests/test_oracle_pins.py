@@ -540,3 +540,31 @@ def test_hit_rate_golden_table():
     lines = [ln.strip() for ln in open(os.path.join(here, "golden", "hit_rates.txt")) if not ln.startswith("#")]
     got = mk.rows(*mk.REGIMES[0])
     assert got == lines[:len(got)]
+
+
+# --------------------------------------------------------------------------
+# COMPACT_KV / ROLLBACK_KV (Alg. 1)
+
+
+def test_compact_kv_hand_example(orc):
+    # one plane, one head, D = 1, positions labelled by their index: prefix
+    # of 3, main chain of K = 2 (positions 3-4), branches of 2 (slot 0 at
+    # 5-6, slot 1 at 7-8, slot 2 at 9-10)
+    kv = np.arange(12, dtype=np.float32).reshape(1, 1, 1, 12, 1).repeat(4, axis=1)
+    al = np.array([0, 1, 2, 1], np.int32)
+    slot = np.array([1, 2, -2, -1], np.int32)
+    out, n = orc.compact_kv(kv, [3, 3, 3, 3], al, slot, 2, 2)
+    assert list(n) == [5, 6, 5, 4]
+    assert out[0, 0, 0, :, 0].tolist() == [0, 1, 2, 7, 8, 5, 6, 7, 8, 9, 10, 11]    # slot 1 behind t+0
+    assert out[0, 1, 0, :, 0].tolist() == [0, 1, 2, 3, 9, 10, 6, 7, 8, 9, 10, 11]   # slot 2 behind t+1
+    assert (out[0, 2:] == kv[0, 2:]).all()                                          # accept / miss: no move
+
+
+def test_compact_kv_overlapping_move_and_bounds(orc):
+    # branch rows overlap their destination (distance 1 < length 3)
+    kv = np.arange(10, dtype=np.float32).reshape(1, 1, 1, 10, 1)
+    out, n = orc.compact_kv(kv, [2], [1], [0], 2, 3)   # src 4..6 -> dst 3..5
+    assert n[0] == 6
+    assert out[0, 0, 0, :, 0].tolist() == [0, 1, 2, 4, 5, 6, 6, 7, 8, 9]
+    out, n = orc.compact_kv(kv, [6], [0], [0], 2, 3)   # src 8..10 passes the end
+    assert n[0] == -1 and (out == kv).all()
