@@ -238,6 +238,31 @@ aces_status aces_resample_sparse(const int32_t *accept_len, const int32_t *topk_
                                  int32_t *status, aces_stream_t stream);
 
 /*
+ * COMPACT_KV / ROLLBACK_KV of the edge pipeline (Alg. 1; Sec. III-C): after
+ * aces_cache_lookup, realign each sequence's KV cache so that the next cycle
+ * continues from contiguous rows.
+ *   kv [planes, B, H, S, D]  device array of elem_bytes-sized elements
+ *                            (planes = layers x {K, V}); 16-byte aligned,
+ *                            D * elem_bytes a multiple of 16.  Updated in place.
+ * Tree layout of sequence b: its prefix of prefix_len[b] positions, then
+ * the main chain (K positions), then the branches in slot order (the slots
+ * of aces_cache_lookup), branch_len positions each (the branch token and
+ * its drafted continuation).  With pi = accept_len[b] and s = slot[b]:
+ *   s >= 0 (hit):   rows [t+K+s*branch_len, +branch_len) move to [t+pi, ...),
+ *                   new_len[b] = t + pi + branch_len;
+ *   s == -2 (whole chain accepted): nothing moves, new_len[b] = t + K;
+ *   s == -1 (miss, ROLLBACK_KV): nothing moves, new_len[b] = t + pi (the
+ *                   rejected drafts and every branch are dropped).
+ * A sequence whose tree would pass position S, or with t < 0 or pi outside
+ * 0..K, gets new_len[b] = -1 and nothing moves.  Rows outside the moved
+ * block keep their contents.  prefix_len, accept_len, slot, new_len: [B]
+ * int32 device arrays.
+ */
+aces_status aces_compact_kv(void *kv, int elem_bytes, int planes, int B, int H, int S, int D,
+                            const int32_t *prefix_len, const int32_t *accept_len, const int32_t *slot, int K,
+                            int branch_len, int32_t *new_len, aces_stream_t stream);
+
+/*
  * Network-aware tree budget (Sec. IV-B, Eq. for B*(t)): the largest tree
  * size B whose edge drafting time fits in the cloud turnaround,
  * draft_latency_s[B - 1] <= rtt_s + verify_s, capped by B_max.  The host

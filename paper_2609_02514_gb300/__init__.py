@@ -63,12 +63,14 @@ def load():
         lib.aces_cache_build.argtypes = [P, P, P, I, I, I, P, P, P]
         lib.aces_cache_lookup.argtypes = [P, P, I, I, P, P, P, P]
         lib.aces_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P]
+        lib.aces_compact_kv.argtypes = [P, I, I, I, I, I, I, P, P, P, I, I, P, P]
         lib.aces_tree_budget.argtypes = [P, I, ctypes.c_double, ctypes.c_double, I, P]
         lib.aces_branch_alloc.argtypes = [I, I, ctypes.c_double, ctypes.c_double, P]
         lib.aces_status_string.argtypes = [I]
         lib.aces_status_string.restype = ctypes.c_char_p
         for f in (lib.aces_verify, lib.aces_sparsify, lib.aces_cache_build, lib.aces_cache_lookup,
-                  lib.aces_resample_sparse, lib.aces_tree_budget, lib.aces_branch_alloc):
+                  lib.aces_resample_sparse, lib.aces_tree_budget, lib.aces_branch_alloc,
+                  lib.aces_compact_kv):
             f.restype = I
         _lib = lib
         return lib
@@ -260,3 +262,19 @@ def branch_alloc(B_alloc: int, gamma: int, alpha: float, beta: float) -> list:
     F = (ctypes.c_int32 * int(gamma))()
     _check("aces_branch_alloc", lib.aces_branch_alloc(int(B_alloc), int(gamma), float(alpha), float(beta), F))
     return [int(f) for f in F]
+
+
+def compact_kv(kv, prefix_len, accept_len, slot, K: int, branch_len: int, new_len: torch.Tensor | None = None):
+    """COMPACT_KV / ROLLBACK_KV (Alg. 1) in place on kv [planes, B, H, S, D];
+    returns new_len [B] int32."""
+    lib = load()
+    kv = _cuda(kv, "kv")
+    t = _cuda(prefix_len, "prefix_len")
+    al = _cuda(accept_len, "accept_len")
+    sl = _cuda(slot, "slot")
+    planes, B, H, S, D = kv.shape
+    out = new_len if new_len is not None else torch.empty(B, dtype=torch.int32, device=kv.device)
+    code = lib.aces_compact_kv(_p(kv), kv.element_size(), planes, B, H, S, D, _p(t), _p(al), _p(sl), int(K),
+                               int(branch_len), _p(out), _stream(kv.device))
+    _check("aces_compact_kv", code)
+    return out

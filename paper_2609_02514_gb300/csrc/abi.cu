@@ -265,6 +265,22 @@ aces_status aces_resample_sparse(const int32_t *accept_len, const int32_t *topk_
     return ACES_OK;
 }
 
+aces_status aces_compact_kv(void *kv, int elem_bytes, int planes, int B, int H, int S, int D,
+                            const int32_t *prefix_len, const int32_t *accept_len, const int32_t *slot, int K,
+                            int branch_len, int32_t *new_len, aces_stream_t stream) {
+    if (!kv || !prefix_len || !accept_len || !slot || !new_len) return ACES_ERR_INVALID_ARG;
+    if (elem_bytes != 1 && elem_bytes != 2 && elem_bytes != 4 && elem_bytes != 8) return ACES_ERR_INVALID_ARG;
+    if (planes < 1 || B < 1 || H < 1 || S < 1 || D < 1 || K < 1 || K > ACES_MAX_K || branch_len < 1)
+        return ACES_ERR_INVALID_ARG;
+    const size_t row_bytes = (size_t)D * (size_t)elem_bytes;
+    if (row_bytes % 16 != 0 || !aligned16(kv)) return ACES_ERR_INVALID_ARG;
+    if ((long long)B * planes * H > (long long)INT_MAX * 8) return ACES_ERR_INVALID_ARG;
+    if (launch_compact_kv(kv, planes, B, H, S, row_bytes, prefix_len, accept_len, slot, K, branch_len, new_len,
+                          reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return ACES_ERR_CUDA;
+    return ACES_OK;
+}
+
 const char *aces_status_string(aces_status s) {
     switch (s) {
         case ACES_OK: return "ok";

@@ -118,3 +118,20 @@ def _resample(lib, **kw):
 ])
 def test_resample_sparse_rejects_invalid_arguments(lib, kw):
     assert _resample(lib, **kw) == 1
+
+
+def _compact(lib, **kw):
+    a = dict(kv=ctypes.c_void_p(0x10000), eb=2, planes=4, B=2, H=2, S=64, D=64, t=FAKE, al=FAKE, sl=FAKE, K=4,
+             L=5, nl=FAKE, s=None)
+    a.update(kw)
+    return lib.aces_compact_kv(a["kv"], a["eb"], a["planes"], a["B"], a["H"], a["S"], a["D"], a["t"], a["al"],
+                               a["sl"], a["K"], a["L"], a["nl"], a["s"])
+
+
+@pytest.mark.parametrize("kw", [
+    dict(kv=None), dict(t=None), dict(al=None), dict(sl=None), dict(nl=None), dict(eb=3), dict(planes=0),
+    dict(B=0), dict(H=0), dict(S=0), dict(D=0), dict(K=0), dict(K=17), dict(L=0), dict(D=4),
+    dict(kv=ctypes.c_void_p(0x10008)),
+])
+def test_compact_kv_rejects_invalid_arguments(lib, kw):
+    assert _compact(lib, **kw) == 1
