@@ -289,3 +289,41 @@ def compact_kv(kv, prefix_len, accept_len, slot, K: int, branch_len: int):
             total = t + pi
         new_len[b] = total if total <= S else -1
     return kv, new_len
+
+
+def tree_mask(F, K: int, branch_len: int):
+    """Tree attention mask of the packed branch forward (Sec. III-C, Fig. for
+    the tree mask), by walking parent pointers.
+
+    Packed order: the main chain (K tokens), then the branches in slot order
+    (depth 0's F_0 branches first), branch_len tokens each: the alternative
+    token at depth d and its drafted continuation.  A token's parent is the
+    token before it on its path: main token m -> m - 1; the first token of a
+    branch at depth d -> main token d - 1 (none at depth 0); a later branch
+    token -> the one before it in its branch.  mask[q, k] is True when k is q
+    or one of its ancestors (every tree token also sees the whole shared
+    prefix, which the mask leaves out); depth[q] = number of ancestors.
+    """
+    F = [int(f) for f in F]
+    n_branch = sum(F)
+    n = K + n_branch * branch_len
+    parent = [-1] * n
+    for m in range(1, K):
+        parent[m] = m - 1
+    s = 0
+    for d in range(K):
+        for _ in range(F[d]):
+            base = K + s * branch_len
+            parent[base] = d - 1
+            for o in range(1, branch_len):
+                parent[base + o] = base + o - 1
+            s += 1
+    mask = np.zeros((n, n), bool)
+    depth = np.zeros(n, np.int32)
+    for q in range(n):
+        k = q
+        while k >= 0:
+            mask[q, k] = True
+            k = parent[k]
+        depth[q] = int(mask[q].sum()) - 1
+    return mask, depth

@@ -568,3 +568,43 @@ def test_compact_kv_overlapping_move_and_bounds(orc):
     assert out[0, 0, 0, :, 0].tolist() == [0, 1, 2, 4, 5, 6, 6, 7, 8, 9]
     out, n = orc.compact_kv(kv, [6], [0], [0], 2, 3)   # src 8..10 passes the end
     assert n[0] == -1 and (out == kv).all()
+
+
+# --------------------------------------------------------------------------
+# tree attention mask (Sec. III-C)
+
+
+def test_tree_mask_hand_example(orc):
+    # K = 3 main tokens m0 m1 m2; one branch at depth 0 (b0 b0'), one at
+    # depth 1 (b1 b1'); branch_len 2 -> 7 tree tokens
+    mask, depth = orc.tree_mask([1, 1, 0], 3, 2)
+    want = np.array([
+        # m0 m1 m2 b0 b0' b1 b1'
+        [1, 0, 0, 0, 0, 0, 0],   # m0
+        [1, 1, 0, 0, 0, 0, 0],   # m1
+        [1, 1, 1, 0, 0, 0, 0],   # m2
+        [0, 0, 0, 1, 0, 0, 0],   # b0: replaces m0, sees no main token
+        [0, 0, 0, 1, 1, 0, 0],   # b0'
+        [1, 0, 0, 0, 0, 1, 0],   # b1: replaces m1, sees m0
+        [1, 0, 0, 0, 0, 1, 1],   # b1'
+    ], bool)
+    assert (mask == want).all()
+    assert depth.tolist() == [0, 1, 2, 0, 1, 1, 2]
+
+
+def test_tree_mask_invariants(orc):
+    F, K, L = [3, 2, 2, 1, 0, 1], 6, 4
+    mask, depth = orc.tree_mask(F, K, L)
+    n = K + sum(F) * L
+    assert mask.shape == (n, n)
+    assert (np.triu(mask, 1) == 0).all()                  # ancestors come first in the packed order
+    assert (np.diag(mask)).all()
+    assert (mask.sum(1) == depth + 1).all()
+    # a branch token at depth d, offset o sees d main tokens and o + 1 branch tokens
+    s = 0
+    for d in range(K):
+        for _ in range(F[d]):
+            for o in range(L):
+                q = K + s * L + o
+                assert mask[q, :K].sum() == d and mask[q, K:].sum() == o + 1 and depth[q] == d + o
+            s += 1
