@@ -263,6 +263,25 @@ aces_status aces_compact_kv(void *kv, int elem_bytes, int planes, int B, int H, 
                             int branch_len, int32_t *new_len, aces_stream_t stream);
 
 /*
+ * Tree attention mask of the packed branch forward (Sec. III-C): every tree
+ * token attends to the shared prefix (all of it; not part of this mask),
+ * to the main-chain tokens before its branch point (main-path block) and to
+ * its own branch up to itself (suffix-diagonal block).  Packed order: the
+ * main chain (K tokens), then the branches in slot order (depth 0's F_0
+ * branches first, as in aces_cache_build), branch_len tokens each (the
+ * alternative token and its drafted continuation); the same layout as
+ * aces_compact_kv.
+ *   n = aces_tree_tokens(F_host, K, branch_len) = K + sum(F) * branch_len
+ *   mask  [n, ceil(n / 32)] uint32 device: bit j of word w of row q is set
+ *         when tree token q may attend to tree token 32 w + j
+ *   depth [n] int32 device: the token's depth (its position is prefix + depth)
+ * aces_tree_tokens returns -1 for invalid sizes (n above 2^20 included).
+ */
+int aces_tree_tokens(const int32_t *F_host, int K, int branch_len);
+aces_status aces_tree_mask(const int32_t *F_host, int K, int branch_len, uint32_t *mask, int32_t *depth,
+                           aces_stream_t stream);
+
+/*
  * Network-aware tree budget (Sec. IV-B, Eq. for B*(t)): the largest tree
  * size B whose edge drafting time fits in the cloud turnaround,
  * draft_latency_s[B - 1] <= rtt_s + verify_s, capped by B_max.  The host

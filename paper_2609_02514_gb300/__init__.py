@@ -64,13 +64,16 @@ def load():
         lib.aces_cache_lookup.argtypes = [P, P, I, I, P, P, P, P]
         lib.aces_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P]
         lib.aces_compact_kv.argtypes = [P, I, I, I, I, I, I, P, P, P, I, I, P, P]
+        lib.aces_tree_tokens.argtypes = [P, I, I]
+        lib.aces_tree_tokens.restype = I
+        lib.aces_tree_mask.argtypes = [P, I, I, P, P, P]
         lib.aces_tree_budget.argtypes = [P, I, ctypes.c_double, ctypes.c_double, I, P]
         lib.aces_branch_alloc.argtypes = [I, I, ctypes.c_double, ctypes.c_double, P]
         lib.aces_status_string.argtypes = [I]
         lib.aces_status_string.restype = ctypes.c_char_p
         for f in (lib.aces_verify, lib.aces_sparsify, lib.aces_cache_build, lib.aces_cache_lookup,
                   lib.aces_resample_sparse, lib.aces_tree_budget, lib.aces_branch_alloc,
-                  lib.aces_compact_kv):
+                  lib.aces_compact_kv, lib.aces_tree_mask):
             f.restype = I
         _lib = lib
         return lib
@@ -278,3 +281,19 @@ def compact_kv(kv, prefix_len, accept_len, slot, K: int, branch_len: int, new_le
                                int(branch_len), _p(out), _stream(kv.device))
     _check("aces_compact_kv", code)
     return out
+
+
+def tree_mask(F, branch_len: int, device=None):
+    """Tree attention mask (Sec. III-C): mask [n, ceil(n/32)] int32 words (bit
+    j of word w: key 32 w + j allowed) and depth [n] int32 on the device."""
+    lib = load()
+    K = len(F)
+    n = int(lib.aces_tree_tokens(_f_host(F), K, int(branch_len)))
+    if n < 0:
+        raise ValueError("invalid tree shape")
+    dev = torch.device("cuda") if device is None else torch.device(device)
+    mask = torch.empty(n, (n + 31) // 32, dtype=torch.int32, device=dev)
+    depth = torch.empty(n, dtype=torch.int32, device=dev)
+    _check("aces_tree_mask", lib.aces_tree_mask(_f_host(F), K, int(branch_len), _p(mask), _p(depth),
+                                                _stream(dev)))
+    return mask, depth

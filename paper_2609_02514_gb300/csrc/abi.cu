@@ -281,6 +281,30 @@ aces_status aces_compact_kv(void *kv, int elem_bytes, int planes, int B, int H, 
     return ACES_OK;
 }
 
+int aces_tree_tokens(const int32_t *F_host, int K, int branch_len) {
+    if (!F_host || K < 1 || K > ACES_MAX_K || branch_len < 1) return -1;
+    long long n = K;
+    for (int d = 0; d < K; ++d) {
+        if (F_host[d] < 0 || F_host[d] > ACES_MAX_BRANCH) return -1;
+        n += (long long)F_host[d] * branch_len;
+    }
+    return n > (1 << 20) ? -1 : (int)n;
+}
+
+aces_status aces_tree_mask(const int32_t *F_host, int K, int branch_len, uint32_t *mask, int32_t *depth,
+                           aces_stream_t stream) {
+    const int n = aces_tree_tokens(F_host, K, branch_len);
+    if (n < 0 || !mask || !depth) return ACES_ERR_INVALID_ARG;
+    int off[ACES_MAX_K + 1];
+    off[0] = 0;
+    for (int d = 0; d < K; ++d) off[d + 1] = off[d] + F_host[d];
+    const int words = (n + 31) / 32;
+    if (launch_tree_mask(off, K, branch_len, n, words, mask, depth, reinterpret_cast<cudaStream_t>(stream)) !=
+        cudaSuccess)
+        return ACES_ERR_CUDA;
+    return ACES_OK;
+}
+
 const char *aces_status_string(aces_status s) {
     switch (s) {
         case ACES_OK: return "ok";

@@ -450,6 +450,8 @@ aces_status verify_impl(const void *target_logits, aces_dtype dt, const float *d
                         int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
                         aces_stream_t stream);
 cudaError_t launch_cache_build(const CacheArgs &a, bool vec, cudaStream_t s);
+cudaError_t launch_tree_mask(const int *off, int K, int branch_len, int n, int words, uint32_t *mask,
+                             int32_t *depth, cudaStream_t s);
 cudaError_t launch_compact_kv(void *kv, int planes, int B, int H, int S, size_t row_bytes,
                               const int32_t *prefix_len, const int32_t *accept_len, const int32_t *slot, int K,
                               int branch_len, int32_t *new_len, cudaStream_t s);

@@ -135,3 +135,14 @@ def _compact(lib, **kw):
 ])
 def test_compact_kv_rejects_invalid_arguments(lib, kw):
     assert _compact(lib, **kw) == 1
+
+
+def test_tree_tokens_and_mask_validation(lib):
+    F = (ctypes.c_int32 * 3)(1, 1, 0)
+    assert lib.aces_tree_tokens(F, 3, 2) == 7
+    assert lib.aces_tree_tokens(F, 3, 0) == -1
+    assert lib.aces_tree_tokens(None, 3, 2) == -1
+    Fbad = (ctypes.c_int32 * 3)(1, -1, 0)
+    assert lib.aces_tree_tokens(Fbad, 3, 2) == -1
+    assert lib.aces_tree_mask(F, 3, 2, None, FAKE, None) == 1
+    assert lib.aces_tree_mask(F, 3, 0, FAKE, FAKE, None) == 1
