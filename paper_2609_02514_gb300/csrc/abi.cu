@@ -44,14 +44,13 @@ aces_status run_rows(RowArgs &a, aces_dtype dt, cudaStream_t s) {
     const size_t es = elem_size(dt);
     const bool vec = aligned16(a.logits) && ((size_t)a.V * es) % 16 == 0;
     const int nsm = sm_count();
-    if (cudaMemsetAsync(a.ws.fb_count, 0, 16, s) != cudaSuccess) return ACES_ERR_CUDA;
+    if (cudaMemsetAsync(a.ws.fb_count, 0, WS_COUNTERS, s) != cudaSuccess) return ACES_ERR_CUDA;
     const int gc = vec ? rows_fast_gc(dt, a.V) : 0;
     if (gc > 0) {
         const int nch = (int)((size_t)a.V * es / 16);
         a.ng = (nch + gc - 1) / gc;  // sketch groups of gc 16-byte chunks
         const size_t smem = rows_fast_smem(dt, gc, nch);
-        const int pgrid = a.rows < 2 * nsm ? a.rows : 2 * nsm;  // persistent: rows claimed dynamically
-        if (launch_rows_fast(a, dt, gc, smem, pgrid, s) != cudaSuccess) return ACES_ERR_CUDA;
+        if (launch_rows_fast(a, dt, gc, smem, s) != cudaSuccess) return ACES_ERR_CUDA;
         int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
         if (launch_rows_general(a, dt, true, 0, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
     } else {

@@ -312,11 +312,13 @@ struct SegSum {
 constexpr int NSEG_MAX = 16;
 constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual step
 
+constexpr int WS_COUNTERS = 32;  // bytes of path counters at the start of the workspace
 // Workspace layout (all offsets 16-byte aligned)
 struct Workspace {
-    int *fb_count;             // [4]   [0] rows handed to the general path, [1] wait timeouts,
+    int *fb_count;             // [8]   [0] rows handed to the general path, [1] wait timeouts,
                                //       [2] rows certified by the full sketch, [3] rows ordered by
-                               //       bitonic sort (path counters, cleared by every call)
+                               //       bitonic sort, [4] rows the general path finished by radix
+                               //       selection (path counters, cleared by every call)
     RowStat *stats;            // [rows]
     int *acc;                  // [B*K] accept bits
     int *fb_list;              // [rows]
@@ -328,7 +330,7 @@ __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t
 // rows = B*(K+1) target rows; nseq = B sequences with K draft positions (K = 0: sparsify);
 // lists: keep every row's nucleus (up to NUC_CAP ids) for the residual step
 __host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K, bool lists) {
-    size_t b = 16 + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
+    size_t b = WS_COUNTERS + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
                align16((size_t)rows * 4);
     if (K > 0) {
         b += align16((size_t)nseq * NSEG_MAX * sizeof(SegSum)) + align16((size_t)nseq * 4);
@@ -340,7 +342,7 @@ __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, in
     char *p = (char *)base;
     Workspace w;
     w.fb_count = (int *)p;
-    p += 16;
+    p += WS_COUNTERS;
     w.stats = (RowStat *)p;
     p += align16((size_t)rows * sizeof(RowStat));
     w.acc = (int *)p;
@@ -438,7 +440,7 @@ __device__ void timeout_row(const RowArgs &a, int r) {
 // host launchers (defined next to their kernels)
 size_t rows_fast_smem(int dt, int gc, int nch);
 int rows_fast_gc(int dt, int V);
-cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, int grid, cudaStream_t s);
+cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, cudaStream_t s);
 cudaError_t launch_rows_general(const RowArgs &a, int dt, bool vec, int direct, int grid, cudaStream_t s);
 cudaError_t launch_resolve(const ResolveArgs &a, int dt, bool vec, cudaStream_t s);
 // aces_verify with a choice: lists = false runs in ws_bytes(rows, B, K, false)

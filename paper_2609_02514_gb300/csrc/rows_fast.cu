@@ -2,9 +2,9 @@
 // packaging of the target distribution; Sec. V-C: compact payload; the
 // acceptance rule is the modified rejection sampling of Sec. II-A).
 //
-// One CTA of 256 threads per target row r = b*(K+1)+i, three CTAs per SM
-// (up to 80 registers per thread, so that every thread keeps eight 16-byte
-// loads in flight), so that the per-row epilogue of one row overlaps the
+// One CTA of 256 threads per target row r = b*(K+1)+i, four CTAs per SM
+// (64 registers per thread with eight 16-byte loads in flight, and a sketch
+// of at most 16 KB), so that the per-row epilogue of one row overlaps the
 // HBM stream of the others.
 //
 //   pass 1   every logit is read once from HBM with 16-byte loads (eight in
@@ -152,7 +152,7 @@ __device__ __forceinline__ void fallback_row(const RowArgs &a, int r) {
 }
 
 template <int DT, int GC>
-__global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
+__global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     using E = Elem<DT>;
     using SK = typename Sketch<DT>::T;
     constexpr int EPC = E::EPC;
@@ -596,12 +596,14 @@ __global__ void __launch_bounds__(NTF, 3) k_rows_fast(RowArgs a) {
     }
 }
 
-// Chunks per sketch group: the smallest power of two >= 2 that keeps the
+// Chunks per sketch group: the smallest power of two >= 4 that keeps the
 // sketch within SKETCH_CAP groups; 0 when the fast kernel cannot take the row.
+// Four chunks (32 bf16 / 16 fp32 logits) per group keep the sketch at 16 KB
+// for a 256000-id bf16 row, which leaves room for four CTAs per SM.
 int rows_fast_gc(int dt, int V) {
     const int nch = (int)((size_t)V * (dt == ACES_BF16 ? 2 : 4) / 16);
     const int gmax = 8;  // 16 chunks per group would not fit the register budget
-    for (int gc = 2; gc <= gmax; gc *= 2)
+    for (int gc = 4; gc <= gmax; gc *= 2)
         if ((nch + gc - 1) / gc <= SKETCH_CAP) return gc;
     return 0;
 }
@@ -630,9 +632,8 @@ static cudaError_t launch_fast_dt(const RowArgs &a, int gc, size_t smem, cudaStr
     return cudaGetLastError();
 }
 
-// one CTA per row (grid = rows); `grid` is unused
-cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, int grid, cudaStream_t s) {
-    (void)grid;
+// one CTA per row (grid = rows)
+cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, cudaStream_t s) {
     return dt == ACES_BF16 ? launch_fast_dt<ACES_BF16>(a, gc, smem, s) : launch_fast_dt<ACES_F32>(a, gc, smem, s);
 }
 

@@ -1,11 +1,16 @@
 // Exact general row kernel of the AceSpec cloud step (Sec. III-B; Sec. II-A
 // modified rejection sampling; Sec. V-C payload).  It takes every row that
 // the fast kernel cannot certify (and every row when the logits are not
-// 16-byte aligned): exact radix selection over the 64-bit order value
-// O = key(z) << 32 | (2^32 - 1 - id), 8 bits per pass, with masses in 2^-40
-// fixed point so that every partial sum is exact and order-independent.
-// One CTA of 512 threads per row; a persistent grid walks the list of rows
-// handed over by the fast kernel.
+// 16-byte aligned).  Masses are in 2^-40 fixed point, so every partial sum
+// is exact and order-independent.  One CTA of 512 threads per row; a
+// persistent grid walks the list of rows handed over by the fast kernel.
+//   binned path  exact per-bin masses over bins of distance below the max
+//                (warp-aggregated shared-memory atomics, farther elements
+//                summed in registers), then the crossing bin and the payload
+//                bins are collected and sorted: three to four row reads;
+//   radix path   when a needed bin is too full or too far: exact radix
+//                selection over the 64-bit order value
+//                O = key(z) << 32 | (2^32 - 1 - id), 8 bits per pass.
 #include <climits>
 
 #include "common.cuh"
@@ -99,6 +104,49 @@ __device__ __forceinline__ void for_each_elem(const char *row, int V, F f) {
     }
 }
 
+// Warp-uniform walk over the row: every lane of a warp takes part in every
+// round (f gets valid = false past the end), so f may use warp collectives.
+template <int DT, bool VEC, class F>
+__device__ __forceinline__ void for_each_elem_warp(const char *row, int V, F f) {
+    using E = Elem<DT>;
+    if (VEC) {
+        const int nch = V / E::EPC;
+        for (int c0 = threadIdx.x & ~31; c0 < nch; c0 += NT) {
+            const int cc = c0 + (threadIdx.x & 31);
+            const bool in = cc < nch;
+            const uint4 w = in ? ldg16(row + (size_t)cc * 16) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+            for (int e = 0; e < E::EPC; ++e) f(in, cc * E::EPC + e, E::get(w, e));
+        }
+    } else {
+        for (int x0 = threadIdx.x & ~31; x0 < V; x0 += NT) {
+            const int x = x0 + (threadIdx.x & 31);
+            const bool in = x < V;
+            f(in, x, in ? E::load1(row, x) : 0.0f);
+        }
+    }
+}
+
+// cnt[d] += 1 and mass[d] += m for every lane with ok; a warp whose lanes
+// all hit one bin (the common case in the first digits, where the logits
+// share their leading key bits) adds its totals with one atomic each
+__device__ __forceinline__ void hist_add(uint32_t *cnt, unsigned long long *mass, bool ok, int d,
+                                         unsigned long long m, bool with_mass) {
+    const unsigned act = __ballot_sync(0xffffffffu, ok);
+    if (act == 0u) return;
+    const int d0 = __shfl_sync(0xffffffffu, d, __ffs(act) - 1);
+    if (__all_sync(0xffffffffu, !ok || d == d0)) {
+        const unsigned long long ms = with_mass ? warp_sum(ok ? m : 0ull) : 0ull;
+        if ((threadIdx.x & 31) == 0) {
+            atomicAdd(&cnt[d0], (uint32_t)__popc(act));
+            if (with_mass) atomicAdd(&mass[d0], ms);
+        }
+    } else if (ok) {
+        atomicAdd(&cnt[d], 1u);
+        if (with_mass) atomicAdd(&mass[d], m);
+    }
+}
+
 struct SelState {
     uint32_t cnt[256];
     unsigned long long mass[256];
@@ -147,13 +195,13 @@ __device__ unsigned long long radix_select(const char *row, int V, float kref, f
         __syncthreads();
         const unsigned long long prefix = st->prefix;
         const int sh = 64 - nbits;
-        for_each_elem<DT, VEC>(row, V, [&](int x, float v) {
-            if (!(v > -INFINITY)) return;
-            unsigned long long o = order_val(fkey(v), (uint32_t)x);
-            if (nbits != 0 && (o >> sh) != prefix) return;
-            int d = (int)((o >> s) & 255ull);
-            atomicAdd(&st->cnt[d], 1u);
-            if (mode == 0 || want_S) atomicAdd(&st->mass[d], to_fx(ex2(fmaf(v, c, -kref))));
+        const bool with_mass = mode == 0 || want_S;
+        for_each_elem_warp<DT, VEC>(row, V, [&](bool in, int x, float v) {
+            const unsigned long long o = order_val(fkey(v), (uint32_t)x);
+            const bool ok = in && v > -INFINITY && (nbits == 0 || (o >> sh) == prefix);
+            const int d = (int)((o >> s) & 255ull);
+            const unsigned long long m = (ok && with_mass) ? to_fx(ex2(fmaf(v, c, -kref))) : 0ull;
+            hist_add(st->cnt, st->mass, ok, d, m, with_mass);
         });
         __syncthreads();
         if (tid == 0) {
@@ -205,10 +253,195 @@ __device__ unsigned long long radix_select(const char *row, int V, float kref, f
     return st->prefix;
 }
 
+// ---------------------------------------------------------------------------
+// Binned exact selection.  Elements are binned by their distance below the
+// row max, d = (m - z) * inv_w (width T/8, bin 255 = everything farther),
+// with exact fixed-point masses per bin.  Bins are ordered by value, so the
+// nucleus crossing lies in the first bin whose cumulative mass reaches the
+// target, and the first k nucleus ids in the bins up to the one where the
+// cumulative count reaches k.  Those bins' elements are collected (at most
+// GB_CAP each) and ordered in shared memory.  Returns false, having
+// written nothing, when a needed bin is the far bin or too full; the radix
+// selection then finishes the row.
+constexpr int GB_CAP = 2048;
+
+constexpr int GB_WIN = 96;  // bins of the first pass (12 temperatures below the max)
+
+struct BinState {
+    uint32_t cnt[NBIN];              // counts of every bin seen so far
+    unsigned long long mass[NBIN];   // masses of the current window's bins
+    unsigned long long S_fx;         // total mass of the row
+    unsigned long long xs[GB_CAP];  // order values of the crossing bin
+    unsigned long long ps[GB_CAP];  // order values of the payload bins
+    int nx, np_, bx, bk, ok, nbelow;
+    unsigned long long above;       // mass of the bins before the crossing bin
+    double target;
+};
+
+// appends o to arr[*n] for every lane with take (one atomic per warp)
+__device__ __forceinline__ void warp_append(unsigned long long *arr, int *n, bool take, unsigned long long o) {
+    const unsigned bal = __ballot_sync(0xffffffffu, take);
+    if (bal == 0u) return;
+    const int lane = threadIdx.x & 31;
+    int base = 0;
+    if (lane == __ffs(bal) - 1) base = atomicAdd(n, __popc(bal));
+    base = __shfl_sync(0xffffffffu, base, __ffs(bal) - 1);
+    const int pos = base + __popc(bal & ((1u << lane) - 1u));
+    if (take && pos < GB_CAP) arr[pos] = o;
+}
+
+template <int DT, bool VEC>
+__device__ bool binned_row(const RowArgs &a, int r, const char *row, float m, float kref,
+                           unsigned long long n_fin, BinState *bs, unsigned long long *buf, double *redd,
+                           unsigned long long *redu) {
+    const int tid = threadIdx.x;
+    const bool all_in = a.top_p >= 1.0f;
+    // Two windows: the first pass histograms the GB_WIN bins nearest the max
+    // with shared-memory atomics and only sums the farther elements in
+    // registers, so most elements of a peaked row cost no atomic; a second
+    // pass over the remaining bins runs only when the crossing (or the k-th
+    // id) lies farther out.
+    if (tid == 0) {
+        bs->nx = 0;
+        bs->np_ = 0;
+        bs->above = 0ull;
+        bs->nbelow = 0;
+        bs->bx = -2;  // crossing bin, -2 while unknown
+        bs->bk = -2;  // last payload bin, -2 while unknown
+        bs->ok = 1;
+    }
+    for (int i = tid; i < NBIN; i += NT) bs->cnt[i] = 0u;
+    for (int W = 0; W < NBIN - 1; W = W == 0 ? GB_WIN : NBIN - 1) {
+        const int WN = W == 0 ? GB_WIN : NBIN - 1 - W;  // bins of this window
+        for (int i = tid; i < WN; i += NT) bs->mass[i] = 0ull;
+        __syncthreads();
+        unsigned long long far_cnt = 0ull, far_mass = 0ull;
+        for_each_elem_warp<DT, VEC>(row, a.V, [&](bool in, int, float v) {
+            const bool fin = in && v > -INFINITY;
+            const float dd = (m - v) * a.inv_w;
+            const int d = dd < (float)(NBIN - 1) ? (int)dd : NBIN - 1;
+            const bool near = fin && d >= W && d < W + WN && d < NBIN - 1;
+            unsigned long long mf = 0ull;
+            if (fin && d >= W) mf = to_fx(ex2(fmaf(v, a.c, -kref)));
+            if (fin && d >= W && !near) {
+                far_cnt += 1ull;
+                far_mass += mf;
+            }
+            hist_add(bs->cnt + W, bs->mass, near, d - W, mf, true);
+        });
+        far_cnt = block_reduce(far_cnt, redu, SumU64());
+        far_mass = block_reduce(far_mass, redu, SumU64());
+        if (tid == 0) {
+            if (W == 0) {  // the first window sees every element: the total
+                unsigned long long S = far_mass;
+                for (int j = 0; j < WN; ++j) S += bs->mass[j];
+                bs->target = (double)a.top_p * (double)S;
+                bs->S_fx = S;
+            }
+            unsigned long long above = bs->above;
+            int nbelow = bs->nbelow;
+            const int wend = W + WN;
+            if (!all_in && bs->bx == -2) {
+                for (int d = W; d < wend; ++d) {
+                    if ((double)(above + bs->mass[d - W]) >= bs->target) {
+                        bs->bx = d;
+                        break;
+                    }
+                    above += bs->mass[d - W];
+                    nbelow += (int)bs->cnt[d];
+                }
+                bs->above = above;
+                bs->nbelow = nbelow;
+            }
+            // once the nucleus size is bounded, the payload needs min(k, it) ids
+            const bool bx_known = all_in || bs->bx >= 0;
+            if (bx_known && bs->bk == -2) {
+                const long long nnuc_max = all_in ? (long long)n_fin : (long long)bs->nbelow + bs->cnt[bs->bx];
+                const long long want = a.k < nnuc_max ? a.k : nnuc_max;
+                long long c = 0;
+                bs->bk = -1;  // k = 0: no payload
+                for (int d = 0; d < wend && want > 0; ++d) {
+                    c += bs->cnt[d];
+                    if (c >= want) {
+                        bs->bk = d;
+                        break;
+                    }
+                }
+                if (want > 0 && bs->bk < 0) bs->bk = -2;  // farther than this window
+                if (bs->bk >= 0 && c > GB_CAP) bs->ok = 0;
+            }
+            if (bs->bx >= 0 && bs->cnt[bs->bx] > (uint32_t)GB_CAP) bs->ok = 0;
+        }
+        __syncthreads();
+        if (!bs->ok) return false;
+        if ((all_in || bs->bx >= 0) && bs->bk != -2) break;
+    }
+    if ((!all_in && bs->bx < 0) || bs->bk == -2) return false;  // beyond the binned range
+    if (tid == 0 && all_in) bs->bx = -1;
+    __syncthreads();
+    const int bx = bs->bx, bk = bs->bk;
+    // collect the crossing bin and the payload bins
+    for_each_elem_warp<DT, VEC>(row, a.V, [&](bool in, int x, float v) {
+        const bool fin = in && v > -INFINITY;
+        const float dd = (m - v) * a.inv_w;
+        const int d = dd < (float)(NBIN - 1) ? (int)dd : NBIN - 1;
+        const unsigned long long o = order_val(fkey(v), (uint32_t)x);
+        warp_append(bs->xs, &bs->nx, fin && d == bx, o);
+        warp_append(bs->ps, &bs->np_, fin && d <= bk, o);
+    });
+    __syncthreads();
+    const int nx = bs->nx, npl = bs->np_;
+    // order both sets (descending order value)
+    {
+        const int p2 = next_pow2(nx < 2 ? 2 : nx);
+        for (int i = nx + tid; i < p2; i += NT) bs->xs[i] = 0ull;
+        const int q2 = next_pow2(npl < 2 ? 2 : npl);
+        for (int i = npl + tid; i < q2; i += NT) bs->ps[i] = 0ull;
+        __syncthreads();
+        if (bx >= 0) bitonic_sort_desc(bs->xs, p2);
+        if (bk >= 0) bitonic_sort_desc(bs->ps, q2);
+    }
+    // the crossing id: first id of the crossing bin where the cumulative mass reaches the target
+    double S_nuc;
+    unsigned long long cut = 0ull;
+    long long n_nuc;
+    if (bx >= 0) {
+        if (tid == 0) {
+            unsigned long long cum = bs->above;
+            int i = 0;
+            for (; i < nx; ++i) {
+                const unsigned long long mi = to_fx(ex2(fmaf(order_value(bs->xs[i]), a.c, -kref)));
+                if ((double)(cum + mi) >= bs->target) {
+                    cum += mi;
+                    break;
+                }
+                cum += mi;
+            }
+            if (i == nx) i = nx - 1;  // rounding: the bin's last id
+            redd[0] = (double)cum / (double)FX_SCALE;
+            bs->nx = i;  // reuse: position of the crossing in the bin
+        }
+        __syncthreads();
+        S_nuc = redd[0];
+        cut = bs->xs[bs->nx];
+        n_nuc = (long long)bs->nbelow + bs->nx + 1;
+    } else {
+        S_nuc = (double)bs->S_fx / (double)FX_SCALE;
+        n_nuc = (long long)n_fin;
+    }
+    int L = (int)(n_nuc < (long long)a.k ? n_nuc : (long long)a.k);
+    if (L > npl) L = npl;
+    for (int i = tid; i < L; i += NT) buf[i] = bs->ps[i];
+    __syncthreads();
+    finish_row<DT>(a, r, row, kref, S_nuc, cut, all_in ? RS_ALL_IN : 0, buf, L, redd);
+    return true;
+}
+
 template <int DT, bool VEC>
 __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
     using E = Elem<DT>;
     __shared__ SelState st;
+    __shared__ BinState bst;
     __shared__ unsigned long long buf[ACES_MAX_TOPK];
     __shared__ double redd[NWARP];
     __shared__ float redf[NWARP];
@@ -240,6 +473,11 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
             __syncthreads();
             continue;
         }
+        if (binned_row<DT, VEC>(a, r, row, m, kref, n_fin, &bst, buf, redd, redu)) {
+            __syncthreads();
+            continue;
+        }
+        if (tid == 0) atomicAdd(&a.ws.fb_count[4], 1);
         const bool all_in = a.top_p >= 1.0f;
         unsigned long long cut = 0ull;
         double S_nuc;

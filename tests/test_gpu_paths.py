@@ -61,11 +61,11 @@ def _plateau(B, K, V, n_hot, group, seed):
 
 
 def test_second_tier_certification_and_bitonic_order(A, orc):
-    # 1500 near-equal ids in 1500 different groups of 8 float32 logits: the
-    # 512 per-thread top maxima carry too little mass, the full sketch
-    # certifies, and the nucleus (~1200 ids) is ordered by bitonic sort
+    # 1500 near-equal ids in 1500 different sketch groups (16 float32 logits
+    # each): the 512 per-thread top maxima carry too little mass, the full
+    # sketch certifies, and the nucleus (~1200 ids) is ordered by bitonic sort
     w = gen.make_workload(2, 2, 32000, "f32", T=1.0, top_p=0.8, k=64, seed=31)
-    counters, res = _run(A, orc, w, _plateau(2, 2, 32000, 1500, 8, 31))
+    counters, res = _run(A, orc, w, _plateau(2, 2, 32000, 1500, 16, 31))
     fallback, timeouts, second_tier, bitonic = counters
     assert fallback == 0 and timeouts == 0
     assert second_tier == 6 and bitonic == 6, counters
@@ -75,8 +75,8 @@ def test_second_tier_certification_and_bitonic_order(A, orc):
 def test_more_candidates_than_capacity_falls_back(A, orc):
     # 3000 near-equal ids: the nucleus alone exceeds the 2048 candidates the
     # fast kernel holds, so every row goes to the exact general kernel
-    w = gen.make_workload(2, 1, 32000, "f32", T=1.0, top_p=0.8, k=32, seed=32)
-    counters, res = _run(A, orc, w, _plateau(2, 1, 32000, 3000, 8, 32))
+    w = gen.make_workload(2, 1, 64000, "f32", T=1.0, top_p=0.8, k=32, seed=32)
+    counters, res = _run(A, orc, w, _plateau(2, 1, 64000, 3000, 16, 32))
     assert counters[0] == 4, counters
     assert res["checked_seqs"] == 2
 
