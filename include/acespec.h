@@ -139,7 +139,7 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
  * library, kept on every GPU that loads the library until the process exits.
  * This call allocates nothing.
  *   - Size limit: returns ACES_ERR_UNSUPPORTED (nothing launched) when
- *     B > 985 at K = 16, B > 1409 at K = 8, B > 1795 at K = 4 (the limit
+ *     B > 981 at K = 16, B > 1401 at K = 8, B > 1783 at K = 4 (the limit
  *     does not depend on V or k).  The scratch keeps no nucleus lists
  *     unless aces_workspace_bytes(B, K, V, k) fits in it (B <= 14 at
  *     K = 16); without them the residual draw scans its whole row.  The

@@ -44,7 +44,8 @@ aces_status run_rows(RowArgs &a, aces_dtype dt, cudaStream_t s) {
     const size_t es = elem_size(dt);
     const bool vec = aligned16(a.logits) && ((size_t)a.V * es) % 16 == 0;
     const int nsm = sm_count();
-    if (cudaMemsetAsync(a.ws.fb_count, 0, WS_COUNTERS, s) != cudaSuccess) return ACES_ERR_CUDA;
+    const int nseq = a.K > 0 ? a.rows / (a.K + 1) : a.rows;
+    if (cudaMemsetAsync(a.ws.fb_count, 0, ws_clear_bytes(nseq, a.K), s) != cudaSuccess) return ACES_ERR_CUDA;
     const int gc = vec ? rows_fast_gc(dt, a.V) : 0;
     if (gc > 0) {
         const int nch = (int)((size_t)a.V * es / 16);
@@ -111,6 +112,8 @@ aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const fl
     a.tail = tail_mass;
     a.row_status = row_status;
     a.ws = ws_carve(workspace, rows, B, K, lists && top_p < 1.0f);
+    a.accept_len = accept_len;
+    a.out_token = out_token;
     a.ng = 0;
     st = run_rows(a, dt, s);
     if (st != ACES_OK) return st;
@@ -173,6 +176,8 @@ aces_status aces_sparsify(const void *target_logits, aces_dtype dt, int rows, in
     a.tail = tail_mass;
     a.row_status = row_status;
     a.ws = ws_carve(workspace, rows, rows, 0, false);
+    a.accept_len = nullptr;
+    a.out_token = nullptr;
     a.ng = 0;
     return run_rows(a, dt, reinterpret_cast<cudaStream_t>(stream));
 }

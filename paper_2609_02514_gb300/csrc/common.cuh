@@ -323,7 +323,8 @@ struct Workspace {
     int *acc;                  // [B*K] accept bits
     int *fb_list;              // [rows]
     SegSum *seg;               // [B*NSEG_MAX]     (verify only)
-    int *seqdone;              // [B]              (verify only) residual drawn from the list
+    int *seqcnt;               // [B]              (verify only) rows of the sequence finished by the fast kernel
+    int *seqdone;              // [B]              (verify only) token already drawn
     unsigned long long *nuc;   // [rows*NUC_CAP]   (verify with lists) nucleus order values
 };
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
@@ -333,16 +334,29 @@ __host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K, bool lists
     size_t b = WS_COUNTERS + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
                align16((size_t)rows * 4);
     if (K > 0) {
-        b += align16((size_t)nseq * NSEG_MAX * sizeof(SegSum)) + align16((size_t)nseq * 4);
+        b += 2 * align16((size_t)nseq * 4) + align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
         if (lists) b += (size_t)rows * NUC_CAP * 8;
     }
     return b;
+}
+// bytes at the start of the workspace that every call clears: the counters,
+// and for verification the per-sequence row counts and done flags
+__host__ __device__ inline size_t ws_clear_bytes(int nseq, int K) {
+    return WS_COUNTERS + (K > 0 ? 2 * align16((size_t)nseq * 4) : 0);
 }
 __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K, bool lists) {
     char *p = (char *)base;
     Workspace w;
     w.fb_count = (int *)p;
     p += WS_COUNTERS;
+    w.seqcnt = nullptr;
+    w.seqdone = nullptr;
+    if (K > 0) {
+        w.seqcnt = (int *)p;
+        p += align16((size_t)nseq * 4);
+        w.seqdone = (int *)p;
+        p += align16((size_t)nseq * 4);
+    }
     w.stats = (RowStat *)p;
     p += align16((size_t)rows * sizeof(RowStat));
     w.acc = (int *)p;
@@ -350,13 +364,10 @@ __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, in
     w.fb_list = (int *)p;
     p += align16((size_t)rows * 4);
     w.seg = nullptr;
-    w.seqdone = nullptr;
     w.nuc = nullptr;
     if (K > 0) {
         w.seg = (SegSum *)p;
         p += align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
-        w.seqdone = (int *)p;
-        p += align16((size_t)nseq * 4);
         if (lists) w.nuc = (unsigned long long *)p;
     }
     return w;
@@ -375,6 +386,8 @@ struct RowArgs {
     float *topk_probs;
     float *tail;
     int32_t *row_status;
+    int32_t *accept_len;   // verification outputs (null for sparsify)
+    int32_t *out_token;
     Workspace ws;
     int ng;                // sketch groups per row
 };
@@ -402,6 +415,115 @@ struct CacheArgs {
     int32_t *bt;
     float *bp;
 };
+
+// first rejection index pi_b (K when every draft token was accepted)
+__device__ __forceinline__ int first_reject(const Workspace &ws, int b, int K) {
+    int pi = K;
+    for (int i = 0; i < K; ++i)
+        if (!ws.acc[(size_t)b * K + i]) {
+            pi = i;
+            break;
+        }
+    return pi;
+}
+
+struct DrawShared {
+    int pi, bad, tok;
+    unsigned long long thr;
+};
+
+// Residual (pi < K) or bonus (pi = K) draw of sequence b from row pi's stored
+// nucleus (the residual max(0, p - q) is zero outside it): q is read at the
+// nucleus ids only, which are ordered by id, and the token is the smallest id
+// whose prefix sum of 2^-40 fixed-point masses exceeds floor(u * total).
+// Writes accept_len, out_token and seqdone; returns without writing when row
+// pi has no stored nucleus (the scan kernels then draw the sequence).  All
+// NTH threads call it, NTH * 2 >= NUC_CAP; skey, rfx, pfx hold NUC_CAP
+// entries, red NTH / 32.
+template <int NTH>
+__device__ void draw_from_list(const Workspace &ws, const float *q, const float *u, int K, int V, int b,
+                               int32_t *accept_len, int32_t *out_token, int32_t *row_status,
+                               unsigned long long *skey, unsigned long long *rfx, unsigned long long *pfx,
+                               unsigned long long *red, DrawShared *sh) {
+    static_assert(2 * NTH >= NUC_CAP, "two nucleus entries per thread");
+    const int tid = threadIdx.x;
+    if (tid == 0) {
+        sh->pi = first_reject(ws, b, K);
+        sh->bad = 0;
+        sh->tok = -1;
+    }
+    __syncthreads();
+    const int pi = sh->pi;
+    const int r = b * (K + 1) + pi;
+    const RowStat rs = ws.stats[r];
+    if (rs.flags & RS_NONFINITE) {
+        if (tid == 0) {
+            accept_len[b] = pi;
+            out_token[b] = -1;
+            ws.seqdone[b] = 1;
+        }
+        return;
+    }
+    if (rs.nnuc < 0) return;  // no list: the scan kernels draw this sequence
+    const int n = rs.nnuc;
+    const unsigned long long *lst = ws.nuc + (size_t)r * NUC_CAP;
+    const float *qrow = pi < K ? q + ((size_t)b * K + pi) * V : nullptr;
+    const float inv_S = (float)(1.0 / rs.S_nuc);
+    const int np = next_pow2(n < 2 ? 2 : n);
+    for (int i = tid; i < np; i += NTH) {
+        if (i < n) {
+            const unsigned long long o = lst[i];
+            const uint32_t id = order_id(o);
+            const float p = ex2(fmaf(order_value(o), rs.c, -rs.kref)) * inv_S;
+            float rr = p;
+            if (qrow) {
+                const float qx = __ldg(qrow + id);
+                if (!(qx >= 0.0f)) sh->bad = 1;
+                rr = fmaxf(p - qx, 0.0f);
+            }
+            rfx[i] = to_fx(rr);
+            pfx[i] = to_fx(p);
+            skey[i] = ~(((unsigned long long)id << 32) | (unsigned long long)i);
+        } else {
+            skey[i] = 0ull;
+        }
+    }
+    __syncthreads();
+    if (sh->bad) {
+        if (tid == 0) {
+            row_status[r] |= ACES_ROW_BAD_Q;
+            accept_len[b] = pi;
+            out_token[b] = -1;
+            ws.seqdone[b] = 1;
+        }
+        return;
+    }
+    bitonic_sort_desc(skey, np);  // ascending id
+    // two consecutive entries (in id order) per thread
+    const int e0 = 2 * tid, e1 = 2 * tid + 1;
+    const int i0 = e0 < n ? (int)(~skey[e0] & 0xFFFFFFFFull) : -1;
+    const int i1 = e1 < n ? (int)(~skey[e1] & 0xFFFFFFFFull) : -1;
+    const unsigned long long r0 = i0 >= 0 ? rfx[i0] : 0ull, r1 = i1 >= 0 ? rfx[i1] : 0ull;
+    const unsigned long long R = block_reduce_n<NTH>(r0 + r1, red, SumU64());
+    const int mode = R == 0ull;  // p <= q everywhere: draw from p itself
+    const unsigned long long w0 = mode ? (i0 >= 0 ? pfx[i0] : 0ull) : r0;
+    const unsigned long long w1 = mode ? (i1 >= 0 ? pfx[i1] : 0ull) : r1;
+    unsigned long long tot;
+    const unsigned long long ex = block_exscan_n<NTH>(w0 + w1, red, &tot);
+    if (tid == 0) sh->thr = tot > 0ull ? floor_u_times(u[(size_t)b * (K + 1) + K], tot) : 0ull;
+    __syncthreads();
+    const unsigned long long thr = sh->thr;
+    if (tot > 0ull) {
+        if (ex <= thr && thr < ex + w0) sh->tok = (int)(~skey[e0] >> 32);
+        else if (ex + w0 <= thr && thr < ex + w0 + w1) sh->tok = (int)(~skey[e1] >> 32);
+    }
+    __syncthreads();
+    if (tid == 0) {
+        accept_len[b] = pi;
+        out_token[b] = sh->tok;
+        ws.seqdone[b] = 1;
+    }
+}
 
 // Outputs of a row whose logits are not a distribution.
 template <int NTH>

@@ -9,14 +9,15 @@
 // which threads add them; the segment sums of pass one and the prefix scan
 // of pass two therefore agree bit for bit.
 //
-//   k_resolve_list  (B CTAs) when the row kernel kept row pi's nucleus (top_p
-//                   < 1 and at most NUC_CAP ids): the residual max(0, p - q)
-//                   is zero outside the nucleus, so q is read at those ids
-//                   only, they are ordered by id, and the draw is taken from
-//                   their prefix sums.  Identical to the scan below, whose
-//                   other terms are all zero.
-//   k_resolve_seg   (B x nseg CTAs) otherwise: segment sums of the residual
-//                   and of p over the whole row
+//   draw_from_list  (common.cuh; run by the fast row kernel's CTA that
+//                   finishes a sequence's last row) when row pi's nucleus was
+//                   kept (top_p < 1 and at most NUC_CAP ids): the residual
+//                   max(0, p - q) is zero outside the nucleus, so q is read at
+//                   those ids only, they are ordered by id, and the draw is
+//                   taken from their prefix sums.  Identical to the scan
+//                   below, whose other terms are all zero.
+//   k_resolve_seg   (B x nseg CTAs) every other sequence: segment sums of
+//                   the residual and of p over the whole row
 //   k_resolve_pick  (B CTAs) locates the segment holding the draw and scans
 //                   it in 2048-id tiles until the crossing id is found
 #include "common.cuh"
@@ -81,15 +82,6 @@ __device__ __forceinline__ void mass_fx(const char *zrow, const float *qrow, int
     }
 }
 
-__device__ __forceinline__ int first_reject(const Workspace &ws, int b, int K) {
-    int pi = K;
-    for (int i = 0; i < K; ++i)
-        if (!ws.acc[(size_t)b * K + i]) {
-            pi = i;
-            break;
-        }
-    return pi;
-}
 
 template <int DT, bool VEC>
 __global__ void __launch_bounds__(NTR) k_resolve_seg(ResolveArgs a, int nseg, int seglen) {
@@ -243,93 +235,6 @@ __global__ void __launch_bounds__(NTR) k_resolve_pick(ResolveArgs a, int nseg, i
     if (tid == 0) a.out_token[b] = s_tok;
 }
 
-__global__ void __launch_bounds__(NTR) k_resolve_list(ResolveArgs a) {
-    __shared__ unsigned long long skey[NUC_CAP];   // ~(id << 32 | entry), sorted descending
-    __shared__ unsigned long long rfx[NUC_CAP], pfx[NUC_CAP];
-    __shared__ unsigned long long red[NTR / 32];
-    __shared__ int s_pi, s_bad, s_tok;
-    __shared__ unsigned long long s_thr;
-    const int b = blockIdx.x, tid = threadIdx.x;
-    if (tid == 0) {
-        s_pi = first_reject(a.ws, b, a.K);
-        s_bad = 0;
-        s_tok = -1;
-    }
-    __syncthreads();
-    const int pi = s_pi;
-    const int r = b * (a.K + 1) + pi;
-    const RowStat rs = a.ws.stats[r];
-    if (rs.flags & RS_NONFINITE) {
-        if (tid == 0) {
-            a.accept_len[b] = pi;
-            a.out_token[b] = -1;
-            a.ws.seqdone[b] = 1;
-        }
-        return;
-    }
-    if (rs.nnuc < 0) {  // no list: the scan kernels draw this sequence
-        if (tid == 0) a.ws.seqdone[b] = 0;
-        return;
-    }
-    const int n = rs.nnuc;
-    const unsigned long long *lst = a.ws.nuc + (size_t)r * NUC_CAP;
-    const float *qrow = pi < a.K ? a.q + ((size_t)b * a.K + pi) * a.V : nullptr;
-    const float inv_S = (float)(1.0 / rs.S_nuc);
-    const int np = next_pow2(n < 2 ? 2 : n);
-    for (int i = tid; i < np; i += NTR) {
-        if (i < n) {
-            const unsigned long long o = lst[i];
-            const uint32_t id = order_id(o);
-            const float p = ex2(fmaf(order_value(o), rs.c, -rs.kref)) * inv_S;
-            float rr = p;
-            if (qrow) {
-                const float qx = __ldg(qrow + id);
-                if (!(qx >= 0.0f)) s_bad = 1;
-                rr = fmaxf(p - qx, 0.0f);
-            }
-            rfx[i] = to_fx(rr);
-            pfx[i] = to_fx(p);
-            skey[i] = ~(((unsigned long long)id << 32) | (unsigned long long)i);
-        } else {
-            skey[i] = 0ull;
-        }
-    }
-    __syncthreads();
-    if (s_bad) {
-        if (tid == 0) {
-            a.row_status[r] |= ACES_ROW_BAD_Q;
-            a.accept_len[b] = pi;
-            a.out_token[b] = -1;
-            a.ws.seqdone[b] = 1;
-        }
-        return;
-    }
-    bitonic_sort_desc(skey, np);  // ascending id
-    // two consecutive entries (in id order) per thread
-    const int e0 = 2 * tid, e1 = 2 * tid + 1;
-    const int i0 = e0 < n ? (int)(~skey[e0] & 0xFFFFFFFFull) : -1;
-    const int i1 = e1 < n ? (int)(~skey[e1] & 0xFFFFFFFFull) : -1;
-    const unsigned long long r0 = i0 >= 0 ? rfx[i0] : 0ull, r1 = i1 >= 0 ? rfx[i1] : 0ull;
-    const unsigned long long R = block_reduce_n<NTR>(r0 + r1, red, SumU64());
-    const int mode = R == 0ull;  // p <= q everywhere: draw from p itself
-    const unsigned long long w0 = mode ? (i0 >= 0 ? pfx[i0] : 0ull) : r0;
-    const unsigned long long w1 = mode ? (i1 >= 0 ? pfx[i1] : 0ull) : r1;
-    unsigned long long tot;
-    const unsigned long long ex = block_exscan_n<NTR>(w0 + w1, red, &tot);
-    if (tid == 0) s_thr = tot > 0ull ? floor_u_times(a.u[(size_t)b * (a.K + 1) + a.K], tot) : 0ull;
-    __syncthreads();
-    const unsigned long long thr = s_thr;
-    if (tot > 0ull) {
-        if (ex <= thr && thr < ex + w0) s_tok = (int)(~skey[e0] >> 32);
-        else if (ex + w0 <= thr && thr < ex + w0 + w1) s_tok = (int)(~skey[e1] >> 32);
-    }
-    __syncthreads();
-    if (tid == 0) {
-        a.accept_len[b] = pi;
-        a.out_token[b] = s_tok;
-        a.ws.seqdone[b] = 1;
-    }
-}
 
 int resolve_segments(int V) {
     int nseg = (V + 32767) / 32768;
@@ -341,7 +246,6 @@ cudaError_t launch_resolve(const ResolveArgs &a, int dt, bool vec, cudaStream_t 
     int seglen = (a.V + nseg - 1) / nseg;
     seglen = (seglen + EPT - 1) / EPT * EPT;
     const int g1 = a.B * nseg;
-    k_resolve_list<<<a.B, NTR, 0, s>>>(a);
     if (dt == ACES_BF16) {
         if (vec) {
             k_resolve_seg<ACES_BF16, true><<<g1, NTR, 0, s>>>(a, nseg, seglen);

@@ -146,6 +146,30 @@ __device__ __forceinline__ float group_expsum(const uint4 (&w)[GC], float c, flo
     return a + b;
 }
 
+// Called by all threads when this CTA has written row r's outputs and state.
+// The CTA that finishes the last row of a sequence (rows handed to the
+// general kernel are never counted) draws the sequence's token from the
+// stored nucleus, so most sequences need no separate resolve launch.
+template <int NTH>
+__device__ void row_finished(const RowArgs &a, int r, unsigned char *scratch) {
+    if (a.ws.seqcnt == nullptr) return;  // sparsify
+    __shared__ int s_last;
+    __shared__ unsigned long long s_red[NTH / 32];
+    __shared__ DrawShared s_draw;
+    const int b = r / (a.K + 1);
+    __syncthreads();  // every thread's writes of this row are issued
+    if (threadIdx.x == 0) {
+        __threadfence();
+        s_last = atomicAdd(&a.ws.seqcnt[b], 1) == a.K;
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();  // the other rows of the sequence are visible
+    unsigned long long *skey = reinterpret_cast<unsigned long long *>(scratch);
+    draw_from_list<NTH>(a.ws, a.q, a.u, a.K, a.V, b, a.accept_len, a.out_token, a.row_status, skey,
+                        skey + NUC_CAP, skey + 2 * NUC_CAP, s_red, &s_draw);
+}
+
 __device__ __forceinline__ void fallback_row(const RowArgs &a, int r) {
     const int pos = atomicAdd(a.ws.fb_count, 1);
     a.ws.fb_list[pos] = r;
@@ -378,6 +402,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     const int bc = s_bc;
     if (!(S > 0.0 && S < 1e300) || !(m < INFINITY) || !(kref < 1e30f)) {
         nonfinite_row<NTF>(a, r);
+        row_finished<NTF>(a, r, smem);
         return;
     }
     if (bc < 0) {
@@ -594,6 +619,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         rs.nnuc = nnuc;
         a.ws.stats[r] = rs;
     }
+    row_finished<NTF>(a, r, smem);
 }
 
 // Chunks per sketch group: the smallest power of two >= 4 that keeps the
@@ -620,7 +646,6 @@ template <int DT>
 static cudaError_t launch_fast_dt(const RowArgs &a, int gc, size_t smem, cudaStream_t s) {
     void (*fn)(RowArgs) = nullptr;
     switch (gc) {
-        case 2: fn = k_rows_fast<DT, 2>; break;
         case 4: fn = k_rows_fast<DT, 4>; break;
         case 8: fn = k_rows_fast<DT, 8>; break;
         default: break;
