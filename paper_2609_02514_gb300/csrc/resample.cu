@@ -11,14 +11,19 @@
 // uses p^_I alone.  When the nucleus of row pi fits in the payload, tau = 0
 // and the draw is the exact residual draw of aces_verify.
 //
-// One CTA of 256 threads per sequence:
+// One thread-block cluster of 8 CTAs (256 threads each) per sequence:
 //   1. the payload of row pi is sorted by id in shared memory, and its
 //      weights (p^ - q on I) are gathered;
-//   2. only when tau > 0: one pass over q_pi gives q_rest (compensated fp32)
-//      and, once the spread factor is known, a second pass gives the weight
-//      of every 2048-id tile (four tiles' loads in flight per thread);
+//   2. only when tau > 0, the 8 CTAs split q_pi's 2048-id tiles: one pass
+//      gives each CTA's share of q_rest (compensated fp32), combined through
+//      distributed shared memory; once the spread factor is known a second
+//      pass gives the weight of every tile (four tiles' loads in flight per
+//      thread), and the CTA holding the draw rescans its tile.  Otherwise
+//      the first CTA draws alone and the others exit at once;
 //   3. the draw: smallest id j whose prefix sum exceeds floor(u * R), with
 //      every weight an integer in units of 2^-52 (exact, order independent).
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 
 namespace aces {
@@ -29,6 +34,7 @@ constexpr int STILE = NTS * SEPT;      // ids per tile
 constexpr int SPAY = ACES_MAX_TOPK;    // payload entries
 constexpr int STILES = (ACES_MAX_V + STILE - 1) / STILE;
 constexpr int TPI = 4;                 // tiles per round of the q passes
+constexpr int SCL = 8;                 // CTAs per sequence: one thread-block cluster
 
 // floor(x * 2^52) of a float x in [0, 2^11) from its bits (0 for x <= 0 or NaN)
 __device__ __forceinline__ unsigned long long to_fx52(float x) {
@@ -75,32 +81,43 @@ __device__ __forceinline__ void load_q(const float *qr, int V, int x0, float (&q
 }
 
 template <bool VEC>
-__global__ void __launch_bounds__(NTS) k_resample_sparse(SparseArgs a) {
+__global__ void __cluster_dims__(SCL, 1, 1) __launch_bounds__(NTS) k_resample_sparse(SparseArgs a) {
+    namespace cg = cooperative_groups;
     __shared__ unsigned long long skey[SPAY];  // ~(id << 32 | entry), sorted descending
     __shared__ int sid[SPAY];                  // payload ids, ascending
     __shared__ unsigned long long sw[SPAY];    // their weights (2^-52 units)
-    __shared__ unsigned long long tsum[STILES];
+    __shared__ unsigned long long tsum[(STILES + SCL - 1) / SCL];  // this CTA's tiles
     __shared__ unsigned long long red[NTS / 32];
     __shared__ unsigned long long red4[TPI][NTS / 32];
     __shared__ float redh[NTS / 32], redl[NTS / 32];
+    __shared__ float s_ph, s_pl;               // this CTA's share of q_rest (read by the cluster)
+    __shared__ int s_pbad;
     __shared__ int s_n, s_bad, s_tok, s_tile;
     __shared__ float s_gam;
-    __shared__ unsigned long long s_thr, s_base;
-    const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    __shared__ unsigned long long s_thr, s_base, s_R;
+    cg::cluster_group cl = cg::this_cluster();
+    const int rank = (int)cl.block_rank();
+    const int b = blockIdx.x / SCL, tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int R1 = a.K + 1;
     const int pi = a.accept_len[b];
-    if (pi < 0 || pi > a.K || (a.row_status[(size_t)b * R1 + pi] & ACES_ROW_NONFINITE)) {
+    const bool bad_row = pi < 0 || pi > a.K || (a.row_status[(size_t)b * R1 + pi] & ACES_ROW_NONFINITE);
+    const size_t row = (size_t)b * R1 + (bad_row ? 0 : pi);
+    const float tau = a.tail[row];
+    const float *qr = (!bad_row && pi < a.K) ? a.q + ((size_t)b * a.K + pi) * a.V : nullptr;
+    // The whole cluster takes part only when the tail may be spread (pi < K,
+    // tau > 0): every CTA then decides the same way from the same inputs, so
+    // all of them reach every cluster barrier.  Otherwise rank 0 works alone.
+    const bool cluster_work = qr != nullptr && tau > 0.0f;
+    if (!cluster_work && rank != 0) return;
+    if (bad_row) {
         if (tid == 0) {
             a.token[b] = -1;
             a.status[b] = ACES_ROW_NONFINITE;
         }
         return;
     }
-    const size_t row = (size_t)b * R1 + pi;
     const int32_t *I = a.ids + row * a.k;
     const float *P = a.probs + row * a.k;
-    const float tau = a.tail[row];
-    const float *qr = pi < a.K ? a.q + ((size_t)b * a.K + pi) * a.V : nullptr;
     const int V = a.V;
 
     // ---- 1. payload sorted by id, weights on it ----
@@ -139,31 +156,34 @@ __global__ void __launch_bounds__(NTS) k_resample_sparse(SparseArgs a) {
         sw[i] = to_fx52(w);
     }
     __syncthreads();
-    if (s_bad || n == 0) {
-        if (tid == 0) {
+    if (s_bad || n == 0) {  // the same in every CTA of the cluster
+        if (rank == 0 && tid == 0) {
             a.token[b] = -1;
             a.status[b] = s_bad ? ACES_ROW_BAD_Q : 0;
         }
         return;
     }
 
-    // ---- 2. the tail, spread like the draft (pi < K, tau > 0) ----
+    // ---- 2. the tail, spread like the draft (pi < K, tau > 0): the cluster ----
     const int ntile = (V + STILE - 1) / STILE;  // 2048-id tiles
+    const int per = (ntile + SCL - 1) / SCL;     // tiles of each CTA
+    const int t_lo = rank * per < ntile ? rank * per : ntile;
+    const int t_hi = t_lo + per < ntile ? t_lo + per : ntile;
     bool spread = false;
-    if (qr && tau > 0.0f) {
+    if (cluster_work) {
         float hi = 0.0f, lo = 0.0f;  // compensated sum of q outside the payload
         int bad = 0;
-        for (int t0 = 0; t0 < ntile; t0 += TPI) {  // TPI tiles' loads in flight
+        for (int t0 = t_lo; t0 < t_hi; t0 += TPI) {  // TPI tiles' loads in flight
             float qv[TPI][SEPT];
 #pragma unroll
             for (int h = 0; h < TPI; ++h) {
                 const int x0 = (t0 + h) * STILE + tid * SEPT;
-                if (x0 < V) load_q<VEC>(qr, V, x0, qv[h]);
+                if (t0 + h < t_hi && x0 < V) load_q<VEC>(qr, V, x0, qv[h]);
             }
 #pragma unroll
             for (int h = 0; h < TPI; ++h) {
                 const int x0 = (t0 + h) * STILE + tid * SEPT;
-                if (x0 >= V) break;
+                if (t0 + h >= t_hi || x0 >= V) break;
                 int j = lower_bound_id(sid, n, x0);
 #pragma unroll
                 for (int e = 0; e < SEPT; ++e) {
@@ -194,43 +214,59 @@ __global__ void __launch_bounds__(NTS) k_resample_sparse(SparseArgs a) {
             redl[wid] = lo;
         }
         __syncthreads();
+        if (tid == 0) {
+            float h = 0.0f, l = 0.0f;
+            for (int i = 0; i < NTS / 32; ++i) {
+                const float sm = h + redh[i];
+                const float bb = sm - h;
+                l = l + redl[i] + ((h - (sm - bb)) + (redh[i] - bb));
+                h = sm;
+            }
+            s_ph = h;
+            s_pl = l;
+            s_pbad = s_bad;
+        }
+        cl.sync();  // every CTA's share is written
+        if (tid == 0) {  // every CTA sums the shares in rank order: the same value everywhere
+            double qrest = 0.0;
+            int anybad = 0;
+            for (int j = 0; j < SCL; ++j) {
+                qrest += (double)*cl.map_shared_rank(&s_ph, j) + (double)*cl.map_shared_rank(&s_pl, j);
+                anybad |= *cl.map_shared_rank(&s_pbad, j);
+            }
+            const double g = qrest > 0.0 ? (double)tau / qrest - 1.0 : 0.0;
+            s_gam = g > 0.0 ? (float)g : 0.0f;
+            s_bad = anybad;
+        }
+        cl.sync();  // the shares are read before any CTA moves on or exits
         if (s_bad) {
-            if (tid == 0) {
+            if (rank == 0 && tid == 0) {
                 a.token[b] = -1;
                 a.status[b] = ACES_ROW_BAD_Q;
             }
             return;
         }
-        if (tid == 0) {
-            double qrest = 0.0;
-            for (int i = 0; i < NTS / 32; ++i) qrest += (double)redh[i] + (double)redl[i];
-            const double g = qrest > 0.0 ? (double)tau / qrest - 1.0 : 0.0;
-            s_gam = g > 0.0 ? (float)g : 0.0f;
-        }
-        __syncthreads();
         spread = s_gam > 0.0f;
+        if (!spread && rank != 0) return;
     }
 
     // ---- 3. the draw ----
     if (spread) {
         const float gam = s_gam;
-        for (int t = tid; t < ntile; t += NTS) tsum[t] = 0ull;
-        __syncthreads();
-        // weight of every tile: q * gam outside the payload, sw on it;
-        // TPI tiles per round, one block reduction of TPI sums
-        for (int t0 = 0; t0 < ntile; t0 += TPI) {
+        // weight of each of this CTA's tiles: q * gam outside the payload, sw on it
+        for (int t0 = t_lo; t0 < t_hi; t0 += TPI) {
             float qv[TPI][SEPT];
 #pragma unroll
             for (int h = 0; h < TPI; ++h) {
                 const int x0 = (t0 + h) * STILE + tid * SEPT;
-                if (x0 < V) load_q<VEC>(qr, V, x0, qv[h]);
+                if (t0 + h < t_hi && x0 < V) load_q<VEC>(qr, V, x0, qv[h]);
             }
             unsigned long long loc[TPI];
 #pragma unroll
             for (int h = 0; h < TPI; ++h) {
                 const int x0 = (t0 + h) * STILE + tid * SEPT;
                 loc[h] = 0ull;
-                if (x0 >= V) continue;
+                if (t0 + h >= t_hi || x0 >= V) continue;
                 int j = lower_bound_id(sid, n, x0);
 #pragma unroll
                 for (int e = 0; e < SEPT; ++e) {
@@ -246,33 +282,54 @@ __global__ void __launch_bounds__(NTS) k_resample_sparse(SparseArgs a) {
 #pragma unroll
                 for (int h = 0; h < TPI; ++h) red4[h][wid] = loc[h];
             __syncthreads();
-            if (tid < TPI && t0 + tid < ntile) {
+            if (tid < TPI && t0 + tid < t_hi) {
                 unsigned long long ts = 0ull;
                 for (int i = 0; i < NTS / 32; ++i) ts += red4[tid][i];
-                tsum[t0 + tid] = ts;
+                tsum[t0 + tid - t_lo] = ts;
             }
             __syncthreads();
         }
-        if (tid == 0) {
+        cl.sync();  // every CTA's tile weights are written
+        if (tid == 0) {  // the same walk over all tiles in every CTA
             unsigned long long tot = 0ull;
-            for (int t = 0; t < ntile; ++t) tot += tsum[t];
-            if (tot == 0ull) s_tile = -1;  // nothing above 2^-52: draw on the payload
-            const unsigned long long thr = tot > 0ull ? floor_u_times(a.u[(size_t)b * R1 + a.K], tot) : 0ull;
-            unsigned long long base = 0ull;
-            int tt = ntile - 1;
-            for (int t = 0; t < ntile; ++t) {
-                if (base + tsum[t] > thr) {
-                    tt = t;
-                    break;
-                }
-                base += tsum[t];
+            for (int j = 0; j < SCL; ++j) {
+                const int lo_j = j * per < ntile ? j * per : ntile;
+                const int hi_j = lo_j + per < ntile ? lo_j + per : ntile;
+                const unsigned long long *rt = cl.map_shared_rank(tsum, j);
+                for (int t = lo_j; t < hi_j; ++t) tot += rt[t - lo_j];
             }
-            if (tot > 0ull) s_tile = tt;
-            s_base = base;
-            s_thr = thr;
+            s_R = tot;
+            s_tile = -1;
+            if (tot > 0ull) {
+                const unsigned long long thr = floor_u_times(a.u[(size_t)b * R1 + a.K], tot);
+                unsigned long long base = 0ull;
+                int tt = ntile - 1;
+                bool found = false;
+                for (int j = 0; j < SCL && !found; ++j) {
+                    const int lo_j = j * per < ntile ? j * per : ntile;
+                    const int hi_j = lo_j + per < ntile ? lo_j + per : ntile;
+                    const unsigned long long *rt = cl.map_shared_rank(tsum, j);
+                    for (int t = lo_j; t < hi_j; ++t) {
+                        if (base + rt[t - lo_j] > thr) {
+                            tt = t;
+                            found = true;
+                            break;
+                        }
+                        base += rt[t - lo_j];
+                    }
+                }
+                if (tt >= t_lo && tt < t_hi) s_tile = tt;
+                s_base = base;
+                s_thr = thr;
+            }
         }
-        __syncthreads();
-        spread = s_tile >= 0;
+        cl.sync();  // the tile weights are read before any CTA exits
+        if (s_R == 0ull) {  // nothing above 2^-52: rank 0 draws on the payload
+            spread = false;
+            if (rank != 0) return;
+        } else if (s_tile < 0) {
+            return;  // another CTA holds the draw
+        }
     }
     if (spread) {
         const float gam = s_gam;
@@ -353,8 +410,8 @@ cudaError_t launch_resample_sparse(const int32_t *accept_len, const int32_t *ids
     a.k = k;
     a.token = token;
     a.status = status;
-    if (vec) k_resample_sparse<true><<<B, NTS, 0, s>>>(a);
-    else k_resample_sparse<false><<<B, NTS, 0, s>>>(a);
+    if (vec) k_resample_sparse<true><<<B * SCL, NTS, 0, s>>>(a);
+    else k_resample_sparse<false><<<B * SCL, NTS, 0, s>>>(a);
     return cudaGetLastError();
 }
 
