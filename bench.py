@@ -37,9 +37,9 @@ sys.path.insert(0, ROOT)
 METRIC = "verified rows/s and achieved HBM GB/s (fraction of GB300 peak) for verify+sparsify"
 WORKLOAD = "b256_k16_v256000_bf16"
 SWEEP_B = (32, 64, 128, 256)
-# kernels of one step: k_rows_fast, k_rows_general, k_resolve_list,
-# k_resolve_seg, k_resolve_pick (aces_verify), k_cache_build, k_cache_lookup
-KERNELS_PER_STEP = 7
+# kernels of one step: k_rows_fast, k_rows_general, k_resolve_seg,
+# k_resolve_pick (aces_verify), k_cache_build, k_cache_lookup
+KERNELS_PER_STEP = 6
 
 
 # ---------------------------------------------------------------------------
@@ -301,7 +301,7 @@ def cpu_baseline(w, inp):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="acespec", choices=["acespec", "reference"])
     ap.add_argument("--workload", default=WORKLOAD)
@@ -410,7 +410,7 @@ def main():
     parts = {
         "verify_sparsify": {"ms": part_ms["verify_sparsify"], "rows_per_s": rows / (part_ms["verify_sparsify"] * 1e-3),
                             "alg_bytes": vb, "gbs": vb / (part_ms["verify_sparsify"] * 1e-3) / 1e9,
-                            "kernels": ["k_rows_fast", "k_rows_general", "k_resolve_list", "k_resolve_seg",
+                            "kernels": ["k_rows_fast", "k_rows_general", "k_resolve_seg",
                                         "k_resolve_pick"],
                             "rows_on_general_path": fb, "rejecting_sequences": n_rej},
         "cache_build": {"ms": part_ms["cache_build"], "alg_bytes": cb,
@@ -506,7 +506,7 @@ def main():
                           "frac_of_peak": by / (ms * 1e-3) / 1e9 / peak})
 
     # end to end through the public API: pinned host inputs in, results out
-    e2e_steps = args.e2e_steps or args.steps
+    e2e_steps = args.e2e_steps or min(args.steps, 30)
     res_keys = ["accept_len", "out_token", "row_status", "topk_ids", "topk_probs", "tail_mass"]
     host_out = {key: torch.empty_like(out[key], device="cpu").pin_memory() for key in res_keys}
     host_cache = {key: torch.empty_like(cache[key], device="cpu").pin_memory() for key in cache}

@@ -80,10 +80,12 @@ typedef struct CUstream_st *aces_stream_t;
 
 /*
  * Bytes of device scratch that aces_verify (B sequences, K >= 1) or
- * aces_sparsify (B rows, K = 0) needs (about 4.1 KiB per target row for
- * aces_verify, under 100 bytes per row for aces_sparsify).  The caller allocates it, passes it
- * to the call and must not use it while the call's work is in flight; it
- * needs no initialisation.  Returns 0 for invalid sizes.
+ * aces_sparsify (B rows, K = 0) needs: about 4.1 KiB per target row for
+ * aces_verify, under 100 bytes per row for aces_sparsify, plus, for both,
+ * room to split up to 640 rows over several CTAs (about V / 4 + 8.3 KiB per
+ * row; 64 MB in all at B = 256, K = 16, V = 256000).  The caller allocates
+ * it, passes it to the call and must not use it while the call's work is in
+ * flight; it needs no initialisation.  Returns 0 for invalid sizes.
  */
 size_t aces_workspace_bytes(int B, int K, int V, int k);
 
@@ -114,7 +116,8 @@ size_t aces_workspace_bytes(int B, int K, int V, int k);
  * workspace / workspace_bytes: device scratch of at least
  *   aces_workspace_bytes(B, K, V, k) bytes, 16-byte aligned.  It includes
  *   4 KiB per row to keep each row's nucleus (when it has at most 512 ids)
- *   for the residual draw, which then reads q at those ids only.
+ *   for the residual draw, which then reads q at those ids only, and the
+ *   areas through which the CTAs sharing a split row combine their parts.
  * Limits: 1 <= B, 1 <= K <= ACES_MAX_K, 2 <= V <= ACES_MAX_V,
  *   0 <= k <= min(V, ACES_MAX_TOPK).
  */
@@ -140,10 +143,11 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
  * This call allocates nothing.
  *   - Size limit: returns ACES_ERR_UNSUPPORTED (nothing launched) when
  *     B > 981 at K = 16, B > 1401 at K = 8, B > 1783 at K = 4 (the limit
- *     does not depend on V or k).  The scratch keeps no nucleus lists
- *     unless aces_workspace_bytes(B, K, V, k) fits in it (B <= 14 at
- *     K = 16); without them the residual draw scans its whole row.  The
- *     results are the same either way.
+ *     does not depend on V or k).  The scratch keeps nucleus lists only for
+ *     B <= 14 at K = 16 (27 at K = 8, 49 at K = 4); without them the
+ *     residual draw scans its whole row.  It splits rows over CTAs only when
+ *     aces_workspace_bytes(B, K, V, k) fits in it (B <= 3 at K = 16 for
+ *     V = 32000).  The results are the same either way.
  *   - Set-up: the first call on each device looks up the array's device
  *     address (cudaGetSymbolAddress) with that device current; make that
  *     first call before any stream capture on the device.

@@ -45,17 +45,36 @@ aces_status run_rows(RowArgs &a, aces_dtype dt, cudaStream_t s) {
     const bool vec = aligned16(a.logits) && ((size_t)a.V * es) % 16 == 0;
     const int nsm = sm_count();
     const int nseq = a.K > 0 ? a.rows / (a.K + 1) : a.rows;
-    if (cudaMemsetAsync(a.ws.fb_count, 0, ws_clear_bytes(nseq, a.K), s) != cudaSuccess) return ACES_ERR_CUDA;
+    if (cudaMemsetAsync(a.ws.fb_count, 0, ws_clear_bytes(nseq, a.K, a.ws.parts != nullptr), s) != cudaSuccess)
+        return ACES_ERR_CUDA;
     const int gc = vec ? rows_fast_gc(dt, a.V) : 0;
     if (gc > 0) {
         const int nch = (int)((size_t)a.V * es / 16);
         a.ng = (nch + gc - 1) / gc;  // sketch groups of gc 16-byte chunks
         const size_t smem = rows_fast_smem(dt, gc, nch);
+        // Split the rows of the last partial wave (every row of a batch
+        // smaller than one wave) over 2 or 4 CTAs, so the SMs stay busy at
+        // the end of the launch.
+        a.r_full = a.rows;
+        a.P = 1;
+        a.gper = a.ng;
+        const long long slots = (long long)rows_fast_per_sm(dt, gc, smem) * nsm;
+        if (a.ws.parts != nullptr && slots > 0) {
+            const long long rr = a.rows < slots ? a.rows : a.rows % slots;
+            if (rr > 0 && rr <= SPLIT_ROWS_MAX) {
+                a.P = 4 * rr <= slots ? 4 : 2;
+                a.r_full = a.rows - (int)rr;
+                a.gper = (a.ng + a.P - 1) / a.P;
+            }
+        }
         if (launch_rows_fast(a, dt, gc, smem, s) != cudaSuccess) return ACES_ERR_CUDA;
         int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
         if (launch_rows_general(a, dt, true, 0, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
     } else {
         a.ng = 0;
+        a.r_full = a.rows;
+        a.P = 1;
+        a.gper = 0;
         int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
         if (launch_rows_general(a, dt, vec, 1, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
     }
@@ -71,26 +90,26 @@ size_t aces_workspace_bytes(int B, int K, int V, int k) {
         return 0;
     long long rows = (long long)B * (K + 1);
     if (rows > INT_MAX / 2) return 0;
-    return ws_bytes((int)rows, B, K, true);
+    return ws_bytes((int)rows, B, K, true, true, V);
 }
 
 }  // extern "C"
 
-// Results do not depend on `lists`: without them the residual draw scans its
-// whole row instead of the stored nucleus.
+// Results depend on neither `lists` (without them the residual draw scans its
+// whole row instead of the stored nucleus) nor `split`.
 aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const float *draft_probs,
                         const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
                         float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
                         int32_t *topk_ids, float *topk_probs, float *tail_mass,
                         int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
-                        aces_stream_t stream) {
+                        bool split, aces_stream_t stream) {
     if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
     aces_status st = check_rows(target_logits, dt, (long long)B * (K + 1), V, T, top_p, k, false,
                                 topk_ids, topk_probs, tail_mass, row_status);
     if (st != ACES_OK) return st;
     if (!draft_probs || !draft_tokens || !uniforms || !accept_len || !out_token || !workspace)
         return ACES_ERR_INVALID_ARG;
-    if (!aligned16(workspace) || workspace_bytes < ws_bytes(B * (K + 1), B, K, lists))
+    if (!aligned16(workspace) || workspace_bytes < ws_bytes(B * (K + 1), B, K, lists, split, V))
         return ACES_ERR_INVALID_ARG;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     const int rows = B * (K + 1);
@@ -111,7 +130,7 @@ aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const fl
     a.topk_probs = topk_probs;
     a.tail = tail_mass;
     a.row_status = row_status;
-    a.ws = ws_carve(workspace, rows, B, K, lists && top_p < 1.0f);
+    a.ws = ws_carve(workspace, rows, B, K, lists && top_p < 1.0f, split, V);
     a.accept_len = accept_len;
     a.out_token = out_token;
     a.ng = 0;
@@ -146,7 +165,7 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
     if (workspace_bytes < aces_workspace_bytes(B, K, V, k)) return ACES_ERR_INVALID_ARG;
     return verify_impl(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
                        accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status,
-                       workspace, workspace_bytes, true, stream);
+                       workspace, workspace_bytes, true, true, stream);
 }
 
 aces_status aces_sparsify(const void *target_logits, aces_dtype dt, int rows, int V, float T,
@@ -175,7 +194,7 @@ aces_status aces_sparsify(const void *target_logits, aces_dtype dt, int rows, in
     a.topk_probs = topk_probs;
     a.tail = tail_mass;
     a.row_status = row_status;
-    a.ws = ws_carve(workspace, rows, rows, 0, false);
+    a.ws = ws_carve(workspace, rows, rows, 0, false, true, V);
     a.accept_len = nullptr;
     a.out_token = nullptr;
     a.ng = 0;

@@ -318,7 +318,8 @@ struct Workspace {
     int *fb_count;             // [8]   [0] rows handed to the general path, [1] wait timeouts,
                                //       [2] rows certified by the full sketch, [3] rows ordered by
                                //       bitonic sort, [4] rows the general path finished by radix
-                               //       selection (path counters, cleared by every call)
+                               //       selection, [5] rows split over several CTAs (path
+                               //       counters, cleared by every call)
     RowStat *stats;            // [rows]
     int *acc;                  // [B*K] accept bits
     int *fb_list;              // [rows]
@@ -326,25 +327,52 @@ struct Workspace {
     int *seqcnt;               // [B]              (verify only) rows of the sequence finished by the fast kernel
     int *seqdone;              // [B]              (verify only) token already drawn
     unsigned long long *nuc;   // [rows*NUC_CAP]   (verify with lists) nucleus order values
+    int *rowcnt;               // [SPLIT_ROWS_MAX] (split rows) parts finished
+    unsigned char *parts;      // [SPLIT_ROWS_MAX * split_row_bytes(V)] (split rows) partial results
+    size_t part_stride;        // split_row_bytes(V)
 };
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
 // rows = B*(K+1) target rows; nseq = B sequences with K draft positions (K = 0: sparsify);
 // lists: keep every row's nucleus (up to NUC_CAP ids) for the residual step
-__host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K, bool lists) {
+// Rows split over several CTAs (the last partial wave of a large batch, or
+// every row of a small one): at most SPLIT_ROWS_MAX rows per call, in at most
+// SPLIT_P_MAX parts of SPLIT_NT threads.  Per split row the workspace keeps
+// each part's statistics and top group maxima, and the row's sketch.
+constexpr int SPLIT_ROWS_MAX = 640;
+constexpr int SPLIT_P_MAX = 4;
+constexpr int SPLIT_NT = 256;
+struct PartStat {
+    float m, kref;  // the part's max and reference
+    double S;       // its exp-sum against kref
+};
+__host__ __device__ inline size_t split_row_bytes(int V) {
+    // sketch: at most V / 16 + 1 groups of 4 bytes (float32 rows, four chunks per group)
+    return align16((size_t)SPLIT_P_MAX * sizeof(PartStat) + (size_t)SPLIT_P_MAX * 2 * SPLIT_NT * 4 +
+                   ((size_t)V / 16 + 1) * 4);
+}
+__host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K, bool lists, bool split = false,
+                                           int V = 0) {
     size_t b = WS_COUNTERS + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
                align16((size_t)rows * 4);
     if (K > 0) {
         b += 2 * align16((size_t)nseq * 4) + align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
         if (lists) b += (size_t)rows * NUC_CAP * 8;
     }
+    if (split) {
+        const int sr = rows < SPLIT_ROWS_MAX ? rows : SPLIT_ROWS_MAX;
+        b += align16((size_t)SPLIT_ROWS_MAX * 4) + (size_t)sr * split_row_bytes(V);
+    }
     return b;
 }
 // bytes at the start of the workspace that every call clears: the counters,
-// and for verification the per-sequence row counts and done flags
-__host__ __device__ inline size_t ws_clear_bytes(int nseq, int K) {
-    return WS_COUNTERS + (K > 0 ? 2 * align16((size_t)nseq * 4) : 0);
+// for verification the per-sequence row counts and done flags, and the
+// split rows' part counts
+__host__ __device__ inline size_t ws_clear_bytes(int nseq, int K, bool split = false) {
+    return WS_COUNTERS + (K > 0 ? 2 * align16((size_t)nseq * 4) : 0) +
+           (split ? align16((size_t)SPLIT_ROWS_MAX * 4) : 0);
 }
-__host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K, bool lists) {
+__host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K, bool lists,
+                                             bool split = false, int V = 0) {
     char *p = (char *)base;
     Workspace w;
     w.fb_count = (int *)p;
@@ -357,6 +385,13 @@ __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, in
         w.seqdone = (int *)p;
         p += align16((size_t)nseq * 4);
     }
+    w.rowcnt = nullptr;
+    w.parts = nullptr;
+    w.part_stride = split_row_bytes(V);
+    if (split) {
+        w.rowcnt = (int *)p;
+        p += align16((size_t)SPLIT_ROWS_MAX * 4);
+    }
     w.stats = (RowStat *)p;
     p += align16((size_t)rows * sizeof(RowStat));
     w.acc = (int *)p;
@@ -368,8 +403,12 @@ __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, in
     if (K > 0) {
         w.seg = (SegSum *)p;
         p += align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
-        if (lists) w.nuc = (unsigned long long *)p;
+        if (lists) {
+            w.nuc = (unsigned long long *)p;
+            p += (size_t)rows * NUC_CAP * 8;
+        }
     }
+    if (split) w.parts = (unsigned char *)p;
     return w;
 }
 
@@ -390,6 +429,9 @@ struct RowArgs {
     int32_t *out_token;
     Workspace ws;
     int ng;                // sketch groups per row
+    int r_full;            // rows r < r_full take one CTA each; the rest are split
+    int P;                 // parts of a split row (1: none)
+    int gper;              // sketch groups per part
 };
 
 // Arguments of the sequence kernel.
@@ -563,16 +605,19 @@ __device__ void timeout_row(const RowArgs &a, int r) {
 size_t rows_fast_smem(int dt, int gc, int nch);
 int rows_fast_gc(int dt, int V);
 cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, cudaStream_t s);
+int rows_fast_per_sm(int dt, int gc, size_t smem);
 cudaError_t launch_rows_general(const RowArgs &a, int dt, bool vec, int direct, int grid, cudaStream_t s);
 cudaError_t launch_resolve(const ResolveArgs &a, int dt, bool vec, cudaStream_t s);
-// aces_verify with a choice: lists = false runs in ws_bytes(rows, B, K, false)
-// bytes of workspace (no nucleus lists; the residual draw scans its row).
+// aces_verify with two choices, neither of which changes the results: lists =
+// false keeps no nucleus lists (the residual draw scans its row), split =
+// false never splits a row over CTAs; the call then needs
+// ws_bytes(rows, B, K, lists, split, V) bytes of workspace.
 aces_status verify_impl(const void *target_logits, aces_dtype dt, const float *draft_probs,
                         const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
                         float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
                         int32_t *topk_ids, float *topk_probs, float *tail_mass,
                         int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
-                        aces_stream_t stream);
+                        bool split, aces_stream_t stream);
 cudaError_t launch_cache_build(const CacheArgs &a, bool vec, cudaStream_t s);
 cudaError_t launch_tree_mask(const int *off, int K, int branch_len, int n, int words, uint32_t *mask,
                              int32_t *depth, cudaStream_t s);

@@ -196,7 +196,15 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     __shared__ float s_inv_S;
     __shared__ unsigned long long s_cut, s_Snuc_fx, s_cumL_fx;
 
-    const int r = blockIdx.x;
+    static_assert(NTF == SPLIT_NT, "split rows keep two group maxima per thread of SPLIT_NT");
+    // rows r < r_full take one CTA each; each later row takes P CTAs, one per
+    // range of gper sketch groups
+    const bool split = (int)blockIdx.x >= a.r_full;
+    const int sj = split ? (int)blockIdx.x - a.r_full : 0;
+    const int r = split ? a.r_full + sj / a.P : (int)blockIdx.x;
+    const int part = split ? sj % a.P : 0;
+    const int g_lo = split ? part * a.gper : 0;
+    const int g_hi = split ? min(ng, g_lo + a.gper) : ng;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const char *row = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
     const int nch = a.V / EPC;
@@ -226,7 +234,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
 #pragma unroll
             for (int j = 0; j < GC; ++j) {
                 const int cc = g * GC + j;
-                w[h][j] = (!CHK || (g < ng && cc < nch)) ? ldg16(row + (size_t)cc * 16) : make_uint4(NI, NI, NI, NI);
+                w[h][j] = (!CHK || (g < g_hi && cc < nch)) ? ldg16(row + (size_t)cc * 16) : make_uint4(NI, NI, NI, NI);
             }
         }
         float im = -INFINITY;
@@ -239,7 +247,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
                 t2 = fminf(gm, t1);
                 t1 = fmaxf(gm, t1);
             }
-            if (!CHK || g < ng) sketch[g] = Sketch<DT>::enc(fkey(gm));
+            if (!CHK || g < g_hi) sketch[g] = Sketch<DT>::enc(fkey(gm));
         }
         m_t = fmaxf(m_t, im);
         const float gk = im * a.c;
@@ -262,9 +270,10 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         else e_t += (gs[0] - t) + s_t;
         s_t = t;
     };
-    int g0 = tid;
-    for (; g0 + (GPI - 1) * NTF < ngf; g0 += NTF * GPI) step(g0, std::false_type());
-    for (; g0 < ng; g0 += NTF * GPI) step(g0, std::true_type());
+    int g0 = g_lo + tid;
+    const int gf_hi = ngf < g_hi ? ngf : g_hi;  // groups of this CTA without a ragged end
+    for (; g0 + (GPI - 1) * NTF < gf_hi; g0 += NTF * GPI) step(g0, std::false_type());
+    for (; g0 < g_hi; g0 += NTF * GPI) step(g0, std::true_type());
     // dependent loads of the accept test, consumed at the end
     float zx = 0.f, qx = 0.f;
     if (xb >= 0 && xb < a.V) {
@@ -282,7 +291,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     }
     for (int i = tid; i < NBIN; i += NTF) bins[i] = 0u;
     __syncthreads();
-    float m = redf[0], kref = redk[0];
+    float m = redf[0], kref = redk[0];  // this CTA's (the row's unless split)
 #pragma unroll
     for (int i = 1; i < NWF; ++i) {
         m = fmaxf(m, redf[i]);
@@ -304,18 +313,73 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
             redl[wid] = lo;
         }
     }
-    // first tier: bins of the 2 * NTF largest group maxima (two per thread);
-    // they carry a lower bound of the mass above every bin edge as well
-    {
+    if (split) {
+        // Publish this part (max, reference, exp-sum, top group maxima and
+        // its sketch groups); the CTA that finishes the row's last part
+        // gathers the others and runs the rest of the row.  No CTA waits.
+        const int si = r - a.r_full;
+        unsigned char *pr = a.ws.parts + (size_t)si * a.ws.part_stride;
+        PartStat *ps = reinterpret_cast<PartStat *>(pr);
+        float *tops = reinterpret_cast<float *>(pr + SPLIT_P_MAX * sizeof(PartStat));
+        SK *gsk = reinterpret_cast<SK *>(pr + SPLIT_P_MAX * sizeof(PartStat) + (size_t)SPLIT_P_MAX * 2 * NTF * 4);
+        tops[(part * 2 + 0) * NTF + tid] = t1;
+        tops[(part * 2 + 1) * NTF + tid] = t2;
+        for (int g = g_lo + tid; g < g_hi; g += NTF) gsk[g] = sketch[g];
+        __syncthreads();
+        if (tid == 0) {
+            double S = 0.0;
+            for (int i = 0; i < NWF; ++i) S += (double)redh[i] + (double)redl[i];
+            PartStat st;
+            st.m = m;
+            st.kref = kref;
+            st.S = S;
+            ps[part] = st;
+            __threadfence();
+            s_ncand = atomicAdd(&a.ws.rowcnt[si], 1) == a.P - 1;  // s_ncand reused as a flag
+        }
+        __syncthreads();
+        if (!s_ncand) return;  // another part finishes the row
+        __threadfence();       // the other parts are visible
+        if (tid == 0) {
+            atomicAdd(&a.ws.fb_count[5], 1);
+            float mm = -INFINITY, kk = -1e30f;
+            for (int p2 = 0; p2 < a.P; ++p2) {
+                mm = fmaxf(mm, ps[p2].m);
+                kk = fmaxf(kk, ps[p2].kref);
+            }
+            double S = 0.0;  // each part's sum rescaled by an exact power of two
+            for (int p2 = 0; p2 < a.P; ++p2) S += ps[p2].S * (double)pow2_int(fmaxf(ps[p2].kref - kk, -1000.0f));
+            s_S = S;
+            redf[0] = mm;
+            redk[0] = kk;
+        }
+        for (int p2 = 0; p2 < a.P; ++p2) {
+            if (p2 == part) continue;
+            const int lo = p2 * a.gper, hi = min(ng, lo + a.gper);
+            for (int g = lo + tid; g < hi; g += NTF) sketch[g] = gsk[g];
+        }
+        __syncthreads();
+        m = redf[0];
+        kref = redk[0];
+        // first tier over every part's top group maxima
+        for (int i = tid; i < a.P * 2 * NTF; i += NTF) {
+            const float t = tops[i];
+            const float d = (m - t) * a.inv_w;
+            if (d < (float)NBIN) atomicAdd(&bins[(int)d], 1u);
+        }
+        __syncthreads();
+    } else {
+        // first tier: bins of the 2 * NTF largest group maxima (two per
+        // thread); they carry a lower bound of the mass above every bin edge
         const float d1 = (m - t1) * a.inv_w, d2 = (m - t2) * a.inv_w;
         if (d1 < (float)NBIN) atomicAdd(&bins[(int)d1], 1u);
         if (d2 < (float)NBIN) atomicAdd(&bins[(int)d2], 1u);
-    }
-    __syncthreads();
-    if (tid == 0) {
-        double S = 0.0;
-        for (int i = 0; i < NWF; ++i) S += (double)redh[i] + (double)redl[i];
-        s_S = S;
+        __syncthreads();
+        if (tid == 0) {
+            double S = 0.0;
+            for (int i = 0; i < NWF; ++i) S += (double)redh[i] + (double)redl[i];
+            s_S = S;
+        }
     }
     const bool all_in = a.top_p >= 1.0f;
     for (int pass = 0; pass < 2; ++pass) {
@@ -653,11 +717,31 @@ static cudaError_t launch_fast_dt(const RowArgs &a, int gc, size_t smem, cudaStr
     if (!fn) return cudaErrorInvalidValue;
     const cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    fn<<<a.rows, NTF, smem, s>>>(a);
+    const long long grid = (long long)a.r_full + (long long)(a.rows - a.r_full) * a.P;
+    fn<<<(unsigned)grid, NTF, smem, s>>>(a);
     return cudaGetLastError();
 }
 
-// one CTA per row (grid = rows)
+template <int DT>
+static int per_sm_dt(int gc, size_t smem) {
+    void (*fn)(RowArgs) = nullptr;
+    switch (gc) {
+        case 4: fn = k_rows_fast<DT, 4>; break;
+        case 8: fn = k_rows_fast<DT, 8>; break;
+        default: return 0;
+    }
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) return 0;
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, NTF, smem) != cudaSuccess) return 0;
+    return n;
+}
+
+// resident CTAs per SM of the fast row kernel (0 when unknown)
+int rows_fast_per_sm(int dt, int gc, size_t smem) {
+    return dt == ACES_BF16 ? per_sm_dt<ACES_BF16>(gc, smem) : per_sm_dt<ACES_F32>(gc, smem);
+}
+
+// one CTA per row r < r_full, P CTAs per later row
 cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, cudaStream_t s) {
     return dt == ACES_BF16 ? launch_fast_dt<ACES_BF16>(a, gc, smem, s) : launch_fast_dt<ACES_F32>(a, gc, smem, s);
 }
