@@ -51,6 +51,34 @@ __device__ __forceinline__ float order_value(unsigned long long o) {
     return fkey_inv((uint32_t)(o >> 32));
 }
 
+// ---------------------------------------------------------------------------
+// Programmatic dependent launch inside one call: a kernel launched with
+// launch_after() is scheduled once every CTA of the previous kernel of the
+// stream has exited or executed pdl_trigger(), without waiting for that
+// kernel's completion and memory flush.  Every CTA of such a kernel executes
+// pdl_wait() before it reads anything the previous kernel wrote (and before
+// it exits, so that its completion implies the previous kernel's).  The fast
+// row kernel never triggers early: general-kernel CTAs placed on the first
+// SMs its last wave frees would crowd there and unbalance that persistent
+// grid.  Without the launch attribute both calls are no-ops.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... P, typename... A>
+inline cudaError_t launch_after(void (*fn)(P...), unsigned grid, unsigned block, cudaStream_t s, A... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, fn, args...);
+}
+
 // 2^x on the special-function unit
 __device__ __forceinline__ float ex2(float x) {
     float y;

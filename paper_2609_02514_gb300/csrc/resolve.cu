@@ -90,6 +90,7 @@ __global__ void __launch_bounds__(NTR) k_resolve_seg(ResolveArgs a, int nseg, in
     __shared__ unsigned long long red[NTR / 32];
     __shared__ int s_bad;
     const int b = blockIdx.x / nseg, sg = blockIdx.x % nseg, tid = threadIdx.x;
+    pdl_wait();  // the row kernels are complete
     if (a.ws.seqdone[b]) return;  // drawn from row pi's nucleus list
     if (tid == 0) {
         const int pi = first_reject(a.ws, b, a.K);
@@ -135,6 +136,7 @@ __global__ void __launch_bounds__(NTR) k_resolve_pick(ResolveArgs a, int nseg, i
     __shared__ unsigned long long s_base, s_thr;
     __shared__ int s_mode, s_pi;
     const int b = blockIdx.x, tid = threadIdx.x;
+    pdl_wait();  // the segment sums are complete
     if (a.ws.seqdone[b]) return;  // drawn from row pi's nucleus list
     if (tid == 0) {
         s_pi = first_reject(a.ws, b, a.K);
@@ -241,29 +243,23 @@ int resolve_segments(int V) {
     return nseg < 1 ? 1 : (nseg > NSEG_MAX ? NSEG_MAX : nseg);
 }
 
+// Both kernels follow the row kernels of the same call and overlap their drain.
 cudaError_t launch_resolve(const ResolveArgs &a, int dt, bool vec, cudaStream_t s) {
     const int nseg = resolve_segments(a.V);
     int seglen = (a.V + nseg - 1) / nseg;
     seglen = (seglen + EPT - 1) / EPT * EPT;
     const int g1 = a.B * nseg;
+    void (*seg)(ResolveArgs, int, int), (*pick)(ResolveArgs, int, int);
     if (dt == ACES_BF16) {
-        if (vec) {
-            k_resolve_seg<ACES_BF16, true><<<g1, NTR, 0, s>>>(a, nseg, seglen);
-            k_resolve_pick<ACES_BF16, true><<<a.B, NTR, 0, s>>>(a, nseg, seglen);
-        } else {
-            k_resolve_seg<ACES_BF16, false><<<g1, NTR, 0, s>>>(a, nseg, seglen);
-            k_resolve_pick<ACES_BF16, false><<<a.B, NTR, 0, s>>>(a, nseg, seglen);
-        }
+        seg = vec ? k_resolve_seg<ACES_BF16, true> : k_resolve_seg<ACES_BF16, false>;
+        pick = vec ? k_resolve_pick<ACES_BF16, true> : k_resolve_pick<ACES_BF16, false>;
     } else {
-        if (vec) {
-            k_resolve_seg<ACES_F32, true><<<g1, NTR, 0, s>>>(a, nseg, seglen);
-            k_resolve_pick<ACES_F32, true><<<a.B, NTR, 0, s>>>(a, nseg, seglen);
-        } else {
-            k_resolve_seg<ACES_F32, false><<<g1, NTR, 0, s>>>(a, nseg, seglen);
-            k_resolve_pick<ACES_F32, false><<<a.B, NTR, 0, s>>>(a, nseg, seglen);
-        }
+        seg = vec ? k_resolve_seg<ACES_F32, true> : k_resolve_seg<ACES_F32, false>;
+        pick = vec ? k_resolve_pick<ACES_F32, true> : k_resolve_pick<ACES_F32, false>;
     }
-    return cudaGetLastError();
+    cudaError_t e = launch_after(seg, (unsigned)g1, NTR, s, a, nseg, seglen);
+    if (e != cudaSuccess) return e;
+    return launch_after(pick, (unsigned)a.B, NTR, s, a, nseg, seglen);
 }
 
 }  // namespace aces

@@ -449,6 +449,7 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
     __shared__ int s_bad;
     __shared__ int s_nbuf;
     const int tid = threadIdx.x;
+    pdl_wait();  // after the fast row kernel: its fallback list is complete
     const int nrows = direct ? a.rows : *a.ws.fb_count;
     for (int idx = blockIdx.x; idx < nrows; idx += gridDim.x) {
         const int r = direct ? idx : a.ws.fb_list[idx];
@@ -525,17 +526,19 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
         finish_row<DT>(a, r, row, kref, S_nuc, cut, all_in ? RS_ALL_IN : 0, buf, L, redd);
         __syncthreads();
     }
+    // only now: resolve CTAs waiting beside busy rows would slow them down
+    pdl_trigger();
 }
 
+// direct = 0 follows the fast row kernel and overlaps its drain
 cudaError_t launch_rows_general(const RowArgs &a, int dt, bool vec, int direct, int grid, cudaStream_t s) {
-    if (dt == ACES_BF16) {
-        if (vec) k_rows_general<ACES_BF16, true><<<grid, NT, 0, s>>>(a, direct);
-        else k_rows_general<ACES_BF16, false><<<grid, NT, 0, s>>>(a, direct);
-    } else {
-        if (vec) k_rows_general<ACES_F32, true><<<grid, NT, 0, s>>>(a, direct);
-        else k_rows_general<ACES_F32, false><<<grid, NT, 0, s>>>(a, direct);
+    void (*fn)(RowArgs, int) = dt == ACES_BF16 ? (vec ? k_rows_general<ACES_BF16, true> : k_rows_general<ACES_BF16, false>)
+                                               : (vec ? k_rows_general<ACES_F32, true> : k_rows_general<ACES_F32, false>);
+    if (direct) {
+        fn<<<grid, NT, 0, s>>>(a, direct);
+        return cudaGetLastError();
     }
-    return cudaGetLastError();
+    return launch_after(fn, (unsigned)grid, NT, s, a, direct);
 }
 
 }  // namespace aces
