@@ -244,9 +244,29 @@ __host__ __device__ __forceinline__ int next_pow2(int n) {
     return p;
 }
 
+// 1/S as a float, the same in every kernel: a probability is always
+// e * inv_mass(S) for a mass e, so a row's outputs do not depend on which
+// kernel finished it (and no fp64 divide sits on the row's critical path)
+__device__ __forceinline__ float inv_mass(double S) { return __frcp_rn((float)S); }
+
+// atomicAdd that releases this CTA's earlier writes (ordered before it by a
+// __syncthreads) and acquires those released by earlier adds to *p
+__device__ __forceinline__ int atomic_add_acq_rel(int *p, int v) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
 // fixed point for exact, order-independent sums of probabilities: floor(x * 2^40)
 // for 0 <= x < 2^23, from the float's bits with integer operations only
 constexpr float FX_SCALE = 1099511627776.0f;  // 2^40
+constexpr double FX_INV = 1.0 / 1099511627776.0;  // 2^-40
+
+// Accept test of Sec. II-A, u < min(1, p/q) with p = e / S, written without
+// a divide: for u < 1 it is u * q * S < e (q > 0).
+__device__ __forceinline__ int accept_test(float u, float q, float e, double S) {
+    return u < 1.0f && (double)u * (double)q * S < (double)e;
+}
 __device__ __forceinline__ unsigned long long to_fx(float x) {
     const uint32_t u = __float_as_uint(x);
     const uint32_t be = u >> 23;                      // biased exponent (sign is 0)
@@ -538,7 +558,7 @@ __device__ void draw_from_list(const Workspace &ws, const float *q, const float 
     const int n = rs.nnuc;
     const unsigned long long *lst = ws.nuc + (size_t)r * NUC_CAP;
     const float *qrow = pi < K ? q + ((size_t)b * K + pi) * V : nullptr;
-    const float inv_S = (float)(1.0 / rs.S_nuc);
+    const float inv_S = inv_mass(rs.S_nuc);
     const int np = next_pow2(n < 2 ? 2 : n);
     for (int i = tid; i < np; i += NTH) {
         if (i < n) {

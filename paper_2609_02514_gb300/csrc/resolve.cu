@@ -109,7 +109,7 @@ __global__ void __launch_bounds__(NTR) k_resolve_seg(ResolveArgs a, int nseg, in
     }
     const char *zrow = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
     const float *qrow = pi < a.K ? a.q + ((size_t)b * a.K + pi) * a.V : nullptr;
-    const float inv_S = (float)(1.0 / rs.S_nuc);
+    const float inv_S = inv_mass(rs.S_nuc);
     const int x_lo = sg * seglen, x_hi = min(a.V, x_lo + seglen);
     unsigned long long sr = 0ull, sp = 0ull;
     int bad = 0;
@@ -198,7 +198,7 @@ __global__ void __launch_bounds__(NTR) k_resolve_pick(ResolveArgs a, int nseg, i
     }
     const char *zrow = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
     const float *qrow = pi < a.K ? a.q + ((size_t)b * a.K + pi) * a.V : nullptr;
-    const float inv_S = (float)(1.0 / rs.S_nuc);
+    const float inv_S = inv_mass(rs.S_nuc);
     const int mode = s_mode;
     const unsigned long long thr = s_thr;
     const int x_lo = s_seg * seglen, x_hi = min(a.V, x_lo + seglen);

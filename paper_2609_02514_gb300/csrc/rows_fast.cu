@@ -158,13 +158,10 @@ __device__ void row_finished(const RowArgs &a, int r, unsigned char *scratch) {
     __shared__ DrawShared s_draw;
     const int b = r / (a.K + 1);
     __syncthreads();  // every thread's writes of this row are issued
-    if (threadIdx.x == 0) {
-        __threadfence();
-        s_last = atomicAdd(&a.ws.seqcnt[b], 1) == a.K;
-    }
+    // releases this row's writes; the last row acquires the others'
+    if (threadIdx.x == 0) s_last = atomic_add_acq_rel(&a.ws.seqcnt[b], 1) == a.K;
     __syncthreads();
     if (!s_last) return;
-    __threadfence();  // the other rows of the sequence are visible
     unsigned long long *skey = reinterpret_cast<unsigned long long *>(scratch);
     draw_from_list<NTH>(a.ws, a.q, a.u, a.K, a.V, b, a.accept_len, a.out_token, a.row_status, skey,
                         skey + NUC_CAP, skey + 2 * NUC_CAP, s_red, &s_draw);
@@ -173,6 +170,15 @@ __device__ void row_finished(const RowArgs &a, int r, unsigned char *scratch) {
 __device__ __forceinline__ void fallback_row(const RowArgs &a, int r) {
     const int pos = atomicAdd(a.ws.fb_count, 1);
     a.ws.fb_list[pos] = r;
+}
+
+// the CTA's exp-sum from the per-warp (hi, lo) pairs, in fp64, by warp 0 (a
+// shuffle tree: three dependent fp64 adds instead of sixteen in one thread)
+__device__ __forceinline__ double warp0_mass(const float *hi, const float *lo, int lane) {
+    double v = lane < NWF ? (double)hi[lane] + (double)lo[lane] : 0.0;
+#pragma unroll
+    for (int o = NWF / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
 }
 
 template <int DT, int GC>
@@ -275,10 +281,11 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     for (; g0 + (GPI - 1) * NTF < gf_hi; g0 += NTF * GPI) step(g0, std::false_type());
     for (; g0 < g_hi; g0 += NTF * GPI) step(g0, std::true_type());
     // dependent loads of the accept test, consumed at the end
-    float zx = 0.f, qx = 0.f;
+    float zx = 0.f, qx = 0.f, ux = 0.f;
     if (xb >= 0 && xb < a.V) {
         zx = E::load1(row, xb);
         qx = __ldg(a.q + ((size_t)bq * a.K + iq) * a.V + xb);
+        ux = __ldg(a.u + (size_t)bq * (a.K + 1) + iq);
     }
 
     // ---- row max, reference and exp-sum (fp32 two-sum tree, fp64 in thread 0) ----
@@ -326,20 +333,21 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         tops[(part * 2 + 1) * NTF + tid] = t2;
         for (int g = g_lo + tid; g < g_hi; g += NTF) gsk[g] = sketch[g];
         __syncthreads();
-        if (tid == 0) {
-            double S = 0.0;
-            for (int i = 0; i < NWF; ++i) S += (double)redh[i] + (double)redl[i];
-            PartStat st;
-            st.m = m;
-            st.kref = kref;
-            st.S = S;
-            ps[part] = st;
-            __threadfence();
-            s_ncand = atomicAdd(&a.ws.rowcnt[si], 1) == a.P - 1;  // s_ncand reused as a flag
+        if (wid == 0) {
+            const double S = warp0_mass(redh, redl, lane);
+            if (lane == 0) {
+                PartStat st;
+                st.m = m;
+                st.kref = kref;
+                st.S = S;
+                ps[part] = st;
+            }
         }
         __syncthreads();
+        // releases this part; the last part acquires the others
+        if (tid == 0) s_ncand = atomic_add_acq_rel(&a.ws.rowcnt[si], 1) == a.P - 1;  // s_ncand reused as a flag
+        __syncthreads();
         if (!s_ncand) return;  // another part finishes the row
-        __threadfence();       // the other parts are visible
         if (tid == 0) {
             atomicAdd(&a.ws.fb_count[5], 1);
             float mm = -INFINITY, kk = -1e30f;
@@ -375,10 +383,9 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         if (d1 < (float)NBIN) atomicAdd(&bins[(int)d1], 1u);
         if (d2 < (float)NBIN) atomicAdd(&bins[(int)d2], 1u);
         __syncthreads();
-        if (tid == 0) {
-            double S = 0.0;
-            for (int i = 0; i < NWF; ++i) S += (double)redh[i] + (double)redl[i];
-            s_S = S;
+        if (wid == 0) {
+            const double S = warp0_mass(redh, redl, lane);
+            if (lane == 0) s_S = S;
         }
     }
     const bool all_in = a.top_p >= 1.0f;
@@ -627,9 +634,9 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
             s_L = L;
             s_Snuc_fx = cN;
             s_cumL_fx = cL;
-            const double sn = all_in ? S : (double)cN / (double)FX_SCALE;
+            const double sn = all_in ? S : (double)cN * FX_INV;
             s_Snuc = sn;
-            s_inv_S = (float)(1.0 / sn);  // one fp64 divide per row
+            s_inv_S = inv_mass(sn);
             s_cut = (nstar != INT_MAX && !all_in) ? ord[nstar] : 0ull;
         }
     }
@@ -657,8 +664,8 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     }
     if (tid == 0) {
         const double S_nuc = s_Snuc;
-        const double cumL = (double)s_cumL_fx / (double)FX_SCALE;
-        if (a.k > 0) a.tail[r] = (float)((S_nuc - cumL) / S_nuc);
+        const double cumL = (double)s_cumL_fx * FX_INV;
+        if (a.k > 0) a.tail[r] = (float)(S_nuc - cumL) * inv_S;
         const unsigned long long cut = s_cut;
         int stt = 0;
         if (a.K > 0 && iq < a.K) {
@@ -667,9 +674,9 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
                 stt |= ACES_ROW_BAD_Q;
             } else {
                 const bool in = all_in ? (zx > -INFINITY) : (order_val(fkey(zx), (uint32_t)xb) >= cut);
-                const double p = in ? (double)ex2(fmaf(zx, a.c, -kref)) / S_nuc : 0.0;
+                const float e = in ? ex2(fmaf(zx, a.c, -kref)) : 0.0f;
                 if (!(qx > 0.0f)) stt |= ACES_ROW_BAD_Q;
-                else accept = (double)a.u[(size_t)bq * (a.K + 1) + iq] < fmin(1.0, p / (double)qx);
+                else accept = accept_test(ux, qx, e, S_nuc);
             }
             a.ws.acc[(size_t)bq * a.K + iq] = accept;
         }

@@ -27,9 +27,9 @@ __device__ void finish_row(const RowArgs &a, int r, const char *row, float kref,
                            int L, double *redd) {
     const int tid = threadIdx.x;
     // same formulas as the fast row kernel, so a row gets bit-identical
-    // outputs whichever kernel finishes it: p = e * (float)(1/S_nuc), and the
+    // outputs whichever kernel finishes it: p = e * inv_mass(S_nuc), and the
     // tail from the exact fixed-point sum of the payload masses
-    const float inv_S = (float)(1.0 / S_nuc);
+    const float inv_S = inv_mass(S_nuc);
     unsigned long long loc = 0ull;
     if (a.k > 0) {
         for (int j = tid; j < a.k; j += NT) {
@@ -49,7 +49,7 @@ __device__ void finish_row(const RowArgs &a, int r, const char *row, float kref,
     __shared__ unsigned long long s_redl[NWARP];
     const unsigned long long tot = block_reduce(loc, s_redl, SumU64());
     if (tid != 0) return;
-    if (a.k > 0) a.tail[r] = (float)((S_nuc - (double)tot / (double)FX_SCALE) / S_nuc);
+    if (a.k > 0) a.tail[r] = (float)(S_nuc - (double)tot * FX_INV) * inv_S;
     int st = 0;
     if (a.K > 0) {
         int b = r / (a.K + 1), i = r % (a.K + 1);
@@ -61,14 +61,10 @@ __device__ void finish_row(const RowArgs &a, int r, const char *row, float kref,
             } else {
                 float v = Elem<DT>::load1(row, x);
                 bool in = (flags & RS_ALL_IN) ? (v > -INFINITY) : (order_val(fkey(v), (uint32_t)x) >= cut);
-                double p = in ? (double)ex2(fmaf(v, a.c, -kref)) / S_nuc : 0.0;
+                const float e = in ? ex2(fmaf(v, a.c, -kref)) : 0.0f;
                 float qx = a.q[((size_t)b * a.K + i) * a.V + x];
-                if (!(qx > 0.0f)) {
-                    st |= ACES_ROW_BAD_Q;
-                } else {
-                    double ratio = p / (double)qx;
-                    accept = (double)a.u[(size_t)b * (a.K + 1) + i] < fmin(1.0, ratio);
-                }
+                if (!(qx > 0.0f)) st |= ACES_ROW_BAD_Q;
+                else accept = accept_test(a.u[(size_t)b * (a.K + 1) + i], qx, e, S_nuc);
             }
             a.ws.acc[(size_t)b * a.K + i] = accept;
         }
@@ -418,7 +414,7 @@ __device__ bool binned_row(const RowArgs &a, int r, const char *row, float m, fl
                 cum += mi;
             }
             if (i == nx) i = nx - 1;  // rounding: the bin's last id
-            redd[0] = (double)cum / (double)FX_SCALE;
+            redd[0] = (double)cum * FX_INV;
             bs->nx = i;  // reuse: position of the crossing in the bin
         }
         __syncthreads();
@@ -426,7 +422,7 @@ __device__ bool binned_row(const RowArgs &a, int r, const char *row, float m, fl
         cut = bs->xs[bs->nx];
         n_nuc = (long long)bs->nbelow + bs->nx + 1;
     } else {
-        S_nuc = (double)bs->S_fx / (double)FX_SCALE;
+        S_nuc = (double)bs->S_fx * FX_INV;
         n_nuc = (long long)n_fin;
     }
     int L = (int)(n_nuc < (long long)a.k ? n_nuc : (long long)a.k);
@@ -485,14 +481,14 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
         unsigned long long n_nuc;
         if (!all_in) {
             cut = radix_select<DT, VEC>(row, a.V, kref, a.c, 0, (double)a.top_p, 0u, true, &st);
-            S_nuc = (double)(st.above + st.found) / (double)FX_SCALE;
+            S_nuc = (double)(st.above + st.found) * FX_INV;
             n_nuc = (unsigned long long)st.above_cnt + 1ull;
         } else {
             unsigned long long sfx = 0ull;
             for_each_elem<DT, VEC>(row, a.V, [&](int, float v) {
                 if (v > -INFINITY) sfx += to_fx(ex2(fmaf(v, a.c, -kref)));
             });
-            S_nuc = (double)block_reduce(sfx, redu, SumU64()) / (double)FX_SCALE;
+            S_nuc = (double)block_reduce(sfx, redu, SumU64()) * FX_INV;
             n_nuc = n_fin;
         }
         __syncthreads();
