@@ -12,8 +12,8 @@
 // and the draw is the exact residual draw of aces_verify.
 //
 // One thread-block cluster of 8 CTAs (256 threads each) per sequence:
-//   1. the payload of row pi is sorted by id in shared memory, and its
-//      weights (p^ - q on I) are gathered;
+//   1. the payload of row pi is ordered by id in shared memory (direct rank
+//      counting), and its weights (p^ - q on I) are gathered;
 //   2. only when tau > 0, the 8 CTAs split q_pi's 2048-id tiles: one pass
 //      gives each CTA's share of q_rest (compensated fp32), combined through
 //      distributed shared memory; once the spread factor is known a second
@@ -83,8 +83,9 @@ __device__ __forceinline__ void load_q(const float *qr, int V, int x0, float (&q
 template <bool VEC>
 __global__ void __cluster_dims__(SCL, 1, 1) __launch_bounds__(NTS) k_resample_sparse(SparseArgs a) {
     namespace cg = cooperative_groups;
-    __shared__ unsigned long long skey[SPAY];  // ~(id << 32 | entry), sorted descending
-    __shared__ int sid[SPAY];                  // payload ids, ascending
+    __shared__ unsigned long long skey[SPAY];  // id << 32 | entry (all ones: invalid id)
+    __shared__ int sid[SPAY];                  // valid payload ids, ascending
+    __shared__ int sidx[SPAY];                 // their payload entries
     __shared__ unsigned long long sw[SPAY];    // their weights (2^-52 units)
     __shared__ unsigned long long tsum[(STILES + SCL - 1) / SCL];  // this CTA's tiles
     __shared__ unsigned long long red[NTS / 32];
@@ -121,7 +122,8 @@ __global__ void __cluster_dims__(SCL, 1, 1) __launch_bounds__(NTS) k_resample_sp
     const int V = a.V;
 
     // ---- 1. payload sorted by id, weights on it ----
-    const int np = next_pow2(a.k < 2 ? 2 : a.k);
+    // The valid entries (0 <= id < V) are ordered by (id, entry) by direct
+    // rank counting: one pass, no barrier stages.
     if (tid == 0) {
         s_n = 0;
         s_bad = 0;
@@ -129,24 +131,26 @@ __global__ void __cluster_dims__(SCL, 1, 1) __launch_bounds__(NTS) k_resample_sp
         s_tile = -1;
         s_gam = 0.0f;
     }
-    for (int j = tid; j < np; j += NTS) {
-        unsigned long long key = 0ull;
-        if (j < a.k) {
-            const int x = I[j];
-            if (x >= 0 && x < V) key = ~(((unsigned long long)x << 32) | (unsigned long long)j);
-        }
+    for (int j = tid; j < a.k; j += NTS) {
+        unsigned long long key = ~0ull;  // invalid: after every valid key
+        const int x = I[j];
+        if (x >= 0 && x < V) key = ((unsigned long long)x << 32) | (unsigned long long)j;
         skey[j] = key;
     }
     __syncthreads();
-    bitonic_sort_desc(skey, np);  // valid entries first, by ascending id
-    for (int j = tid; j < np; j += NTS)
-        if (skey[j] != 0ull && (j + 1 == np || skey[j + 1] == 0ull)) s_n = j + 1;
+    for (int j = tid; j < a.k; j += NTS) {
+        const unsigned long long key = skey[j];
+        if (key == ~0ull) continue;
+        int rank = 0;
+        for (int i = 0; i < a.k; ++i) rank += skey[i] < key;
+        sid[rank] = (int)(key >> 32);
+        sidx[rank] = (int)(key & 0xFFFFFFFFull);
+        atomicAdd(&s_n, 1);
+    }
     __syncthreads();
     const int n = s_n;
     for (int i = tid; i < n; i += NTS) {
-        const unsigned long long kk = ~skey[i];
-        const int x = (int)(kk >> 32), j = (int)(kk & 0xFFFFFFFFull);
-        sid[i] = x;
+        const int x = sid[i], j = sidx[i];
         float w = fmaxf(P[j], 0.0f);
         if (qr) {
             const float qx = __ldg(qr + x);
@@ -372,10 +376,7 @@ __global__ void __cluster_dims__(SCL, 1, 1) __launch_bounds__(NTS) k_resample_sp
         unsigned long long ex = block_exscan_n<NTS>(w, red, &tot);
         if (tot == 0ull) {  // p^ <= q wherever it is known: draw from p^ on the payload
             __syncthreads();
-            if (tid < n) {
-                const int j = (int)(~skey[tid] & 0xFFFFFFFFull);
-                sw[tid] = to_fx52(fmaxf(P[j], 0.0f));
-            }
+            if (tid < n) sw[tid] = to_fx52(fmaxf(P[sidx[tid]], 0.0f));
             __syncthreads();
             w = tid < n ? sw[tid] : 0ull;
             ex = block_exscan_n<NTS>(w, red, &tot);
