@@ -197,6 +197,29 @@ aces_status aces_cache_build(const float *draft_probs, const int32_t *draft_toke
                              float *branch_prob, aces_stream_t stream);
 
 /*
+ * The cloud side of one speculation cycle in one call (Sec. III-B/C;
+ * Algorithm 1): aces_verify and aces_cache_build of the same batch, with the
+ * arguments, outputs, limits and errors of both.  The workspace must hold
+ * aces_workspace_bytes(B, K, V, k) bytes.  The two stream different tensors
+ * (the logits and the draft distributions), so the cache build runs on a
+ * stream of the library's own, forked from `stream` (it waits for the work
+ * queued there before the call) and joined back to it (work queued on
+ * `stream` after the call waits for both).  Results are bit-identical to the
+ * two separate calls.
+ *   - Arguments of both calls are checked before anything is launched.
+ *   - The first call on each device creates that stream and two events
+ *     (kept until the process exits); make it before any stream capture on
+ *     the device.  Calls from several host threads are serialised while they
+ *     queue their work.
+ */
+aces_status aces_cloud_step(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                            const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                            float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                            int32_t *topk_ids, float *topk_probs, float *tail_mass, int32_t *row_status,
+                            const int32_t *F_host, int32_t *branch_tok, float *branch_prob, void *workspace,
+                            size_t workspace_bytes, aces_stream_t stream);
+
+/*
  * O(1) state recovery lookup (Sec. III-B, Algorithm 1: w = (pi, x_resampled),
  * w in dom(T)).  For each sequence: slot[b] = off_pi + j when
  * branch_tok[b, off_pi + j] == token[b] (the first such j); -1 on a miss or

@@ -61,6 +61,7 @@ def load():
         lib.aces_verify.argtypes = [P, I, P, P, P, I, I, I, F, F, P, P, I, P, P, P, P, P, S, P]
         lib.aces_sparsify.argtypes = [P, I, I, I, F, F, I, P, P, P, P, P, S, P]
         lib.aces_cache_build.argtypes = [P, P, P, I, I, I, P, P, P]
+        lib.aces_cloud_step.argtypes = [P, I, P, P, P, I, I, I, F, F, P, P, I, P, P, P, P, P, P, P, P, S, P]
         lib.aces_cache_lookup.argtypes = [P, P, I, I, P, P, P, P]
         lib.aces_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P]
         lib.aces_compact_kv.argtypes = [P, I, I, I, I, I, I, P, P, P, I, I, P, P]
@@ -203,6 +204,53 @@ def cache_build(draft_probs, draft_tokens, F, out: dict | None = None):
     code = lib.aces_cache_build(_p(q), _p(xt), _f_host(F), B, K, V, _p(o["branch_tok"]),
                                 _p(o["branch_prob"]), _stream(dev))
     _check("aces_cache_build", code)
+    return o
+
+
+def cloud_step(target_logits, draft_probs, draft_tokens, uniforms, T: float, top_p: float, k: int, F,
+               out: dict | None = None, workspace: torch.Tensor | None = None):
+    """verify() and cache_build() of the same batch in one call (the cache
+    build runs concurrently on the library's own stream).  Returns the keys of
+    both: accept_len, out_token, row_status, the payload when k > 0,
+    branch_tok and branch_prob."""
+    lib = load()
+    z = _cuda(target_logits, "target_logits")
+    q = _cuda(draft_probs, "draft_probs")
+    xt = _cuda(draft_tokens, "draft_tokens")
+    u = _cuda(uniforms, "uniforms")
+    if z.dim() != 3:
+        raise ValueError("target_logits must be [B, K+1, V]")
+    B, R, V = z.shape
+    K = R - 1
+    if q.dtype != torch.float32 or tuple(q.shape) != (B, K, V):
+        raise ValueError("draft_probs must be float32 [B, K, V]")
+    if xt.dtype != torch.int32 or tuple(xt.shape) != (B, K):
+        raise ValueError("draft_tokens must be int32 [B, K]")
+    if u.dtype != torch.float32 or tuple(u.shape) != (B, R):
+        raise ValueError("uniforms must be float32 [B, K+1]")
+    if len(F) != K:
+        raise ValueError("F must have K entries")
+    tot = int(sum(int(f) for f in F))
+    dev = z.device
+    o = {} if out is None else dict(out)
+    i32 = dict(dtype=torch.int32, device=dev)
+    f32 = dict(dtype=torch.float32, device=dev)
+    o.setdefault("accept_len", torch.empty(B, **i32))
+    o.setdefault("out_token", torch.empty(B, **i32))
+    o.setdefault("row_status", torch.empty(B, R, **i32))
+    if k > 0:
+        o.setdefault("topk_ids", torch.empty(B, R, k, **i32))
+        o.setdefault("topk_probs", torch.empty(B, R, k, **f32))
+        o.setdefault("tail_mass", torch.empty(B, R, **f32))
+    o.setdefault("branch_tok", torch.empty(B, tot, **i32))
+    o.setdefault("branch_prob", torch.empty(B, tot, **f32))
+    need = workspace_bytes(B, K, V, k)
+    ws = workspace if workspace is not None else torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
+    code = lib.aces_cloud_step(_p(z), _dtype_code(z), _p(q), _p(xt), _p(u), B, K, V, float(T), float(top_p),
+                               _p(o["accept_len"]), _p(o["out_token"]), int(k), _p(o.get("topk_ids")),
+                               _p(o.get("topk_probs")), _p(o.get("tail_mass")), _p(o["row_status"]), _f_host(F),
+                               _p(o["branch_tok"]), _p(o["branch_prob"]), _p(ws), ws.numel(), _stream(dev))
+    _check("aces_cloud_step", code)
     return o
 
 

@@ -2,6 +2,7 @@
 // workspace carving.  Nothing here allocates memory.
 #include <climits>
 #include <cmath>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -95,14 +96,12 @@ size_t aces_workspace_bytes(int B, int K, int V, int k) {
 
 }  // extern "C"
 
-// Results depend on neither `lists` (without them the residual draw scans its
-// whole row instead of the stored nucleus) nor `split`.
-aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const float *draft_probs,
-                        const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
-                        float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
-                        int32_t *topk_ids, float *topk_probs, float *tail_mass,
-                        int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
-                        bool split, aces_stream_t stream) {
+// The argument checks of aces_verify (nothing is launched).
+static aces_status verify_check(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                                const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                                float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                                int32_t *topk_ids, float *topk_probs, float *tail_mass, int32_t *row_status,
+                                void *workspace, size_t workspace_bytes, bool lists, bool split) {
     if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
     aces_status st = check_rows(target_logits, dt, (long long)B * (K + 1), V, T, top_p, k, false,
                                 topk_ids, topk_probs, tail_mass, row_status);
@@ -111,6 +110,21 @@ aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const fl
         return ACES_ERR_INVALID_ARG;
     if (!aligned16(workspace) || workspace_bytes < ws_bytes(B * (K + 1), B, K, lists, split, V))
         return ACES_ERR_INVALID_ARG;
+    return ACES_OK;
+}
+
+// Results depend on neither `lists` (without them the residual draw scans its
+// whole row instead of the stored nucleus) nor `split`.
+aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                        const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                        float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                        int32_t *topk_ids, float *topk_probs, float *tail_mass,
+                        int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
+                        bool split, aces_stream_t stream) {
+    aces_status st = verify_check(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
+                                  accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status,
+                                  workspace, workspace_bytes, lists, split);
+    if (st != ACES_OK) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     const int rows = B * (K + 1);
     RowArgs a;
@@ -222,23 +236,93 @@ static aces_status fill_cache_args(CacheArgs &c, const int32_t *F_host, int B, i
     return ACES_OK;
 }
 
-aces_status aces_cache_build(const float *draft_probs, const int32_t *draft_tokens,
-                             const int32_t *F_host, int B, int K, int V, int32_t *branch_tok,
-                             float *branch_prob, aces_stream_t stream) {
-    CacheArgs c;
+// The argument checks of aces_cache_build and its kernel arguments.
+static aces_status cache_prepare(CacheArgs &c, const float *draft_probs, const int32_t *draft_tokens,
+                                 const int32_t *F_host, int B, int K, int V, int32_t *branch_tok,
+                                 float *branch_prob) {
     aces_status st = fill_cache_args(c, F_host, B, K, V);
     if (st != ACES_OK) return st;
     if (!draft_probs || !draft_tokens) return ACES_ERR_INVALID_ARG;
-    if (c.total == 0) return ACES_OK;
-    if (!branch_tok || !branch_prob) return ACES_ERR_INVALID_ARG;
+    if (c.total > 0 && (!branch_tok || !branch_prob)) return ACES_ERR_INVALID_ARG;
     c.q = draft_probs;
     c.xt = draft_tokens;
     c.bt = branch_tok;
     c.bp = branch_prob;
-    const bool vec = aligned16(draft_probs) && V % 4 == 0;
-    if (launch_cache_build(c, vec, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
-        return ACES_ERR_CUDA;
     return ACES_OK;
+}
+
+static aces_status cache_launch(const CacheArgs &c, cudaStream_t s) {
+    if (c.total == 0) return ACES_OK;
+    const bool vec = aligned16(c.q) && c.V % 4 == 0;
+    return launch_cache_build(c, vec, s) == cudaSuccess ? ACES_OK : ACES_ERR_CUDA;
+}
+
+// The library's side stream of the current device, with a fork and a join
+// event: created on the first aces_cloud_step on that device and kept until
+// the process exits.  Held under g_side_mu while a call records and waits.
+struct SideStream {
+    cudaStream_t s;
+    cudaEvent_t fork, join;
+};
+constexpr int SIDE_MAX_DEVICES = 64;
+static std::mutex g_side_mu;
+static SideStream g_side[SIDE_MAX_DEVICES];
+static bool g_side_ok[SIDE_MAX_DEVICES];
+
+static aces_status side_stream(SideStream **out) {  // called with g_side_mu held
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= SIDE_MAX_DEVICES) return ACES_ERR_CUDA;
+    if (!g_side_ok[dev]) {
+        SideStream ss;
+        if (cudaStreamCreateWithFlags(&ss.s, cudaStreamNonBlocking) != cudaSuccess) return ACES_ERR_CUDA;
+        if (cudaEventCreateWithFlags(&ss.fork, cudaEventDisableTiming) != cudaSuccess) return ACES_ERR_CUDA;
+        if (cudaEventCreateWithFlags(&ss.join, cudaEventDisableTiming) != cudaSuccess) return ACES_ERR_CUDA;
+        g_side[dev] = ss;
+        g_side_ok[dev] = true;
+    }
+    *out = &g_side[dev];
+    return ACES_OK;
+}
+
+aces_status aces_cache_build(const float *draft_probs, const int32_t *draft_tokens,
+                             const int32_t *F_host, int B, int K, int V, int32_t *branch_tok,
+                             float *branch_prob, aces_stream_t stream) {
+    CacheArgs c;
+    const aces_status st = cache_prepare(c, draft_probs, draft_tokens, F_host, B, K, V, branch_tok, branch_prob);
+    if (st != ACES_OK) return st;
+    return cache_launch(c, reinterpret_cast<cudaStream_t>(stream));
+}
+
+aces_status aces_cloud_step(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                            const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                            float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                            int32_t *topk_ids, float *topk_probs, float *tail_mass, int32_t *row_status,
+                            const int32_t *F_host, int32_t *branch_tok, float *branch_prob, void *workspace,
+                            size_t workspace_bytes, aces_stream_t stream) {
+    aces_status st = verify_check(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
+                                  accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status,
+                                  workspace, workspace_bytes, true, true);
+    if (st != ACES_OK) return st;
+    if (workspace_bytes < aces_workspace_bytes(B, K, V, k)) return ACES_ERR_INVALID_ARG;
+    CacheArgs c;
+    st = cache_prepare(c, draft_probs, draft_tokens, F_host, B, K, V, branch_tok, branch_prob);
+    if (st != ACES_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    std::lock_guard<std::mutex> lock(g_side_mu);
+    SideStream *ss = nullptr;
+    st = side_stream(&ss);
+    if (st != ACES_OK) return st;
+    // fork: the cache build on the side stream after everything before it on `stream`
+    if (cudaEventRecord(ss->fork, s) != cudaSuccess || cudaStreamWaitEvent(ss->s, ss->fork, 0) != cudaSuccess)
+        return ACES_ERR_CUDA;
+    const aces_status sc = cache_launch(c, ss->s);
+    const aces_status sv = verify_impl(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
+                                       accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status,
+                                       workspace, workspace_bytes, true, true, stream);
+    // join: later work on `stream` waits for the cache build (also after a failure)
+    if (cudaEventRecord(ss->join, ss->s) != cudaSuccess || cudaStreamWaitEvent(s, ss->join, 0) != cudaSuccess)
+        return ACES_ERR_CUDA;
+    return sc != ACES_OK ? sc : sv;
 }
 
 aces_status aces_cache_lookup(const int32_t *branch_tok, const int32_t *F_host, int B, int K,

@@ -76,6 +76,28 @@ def test_verify_rejects_invalid_arguments(lib, kw, code):
     assert _verify(lib, **kw) == code
 
 
+def _step(lib, **kw):
+    F = (ctypes.c_int32 * 4)(2, 2, 2, 2)
+    a = dict(z=FAKE, dt=1, q=FAKE, xt=FAKE, u=FAKE, B=2, K=4, V=1000, T=1.0, top_p=0.9, al=FAKE, tok=FAKE,
+             k=8, ids=FAKE, probs=FAKE, tail=FAKE, st=FAKE, F=F, bt=FAKE, bp=FAKE, ws=FAKE, wsb=1 << 20, s=None)
+    a.update(kw)
+    return lib.aces_cloud_step(a["z"], a["dt"], a["q"], a["xt"], a["u"], a["B"], a["K"], a["V"], a["T"],
+                               a["top_p"], a["al"], a["tok"], a["k"], a["ids"], a["probs"], a["tail"], a["st"],
+                               a["F"], a["bt"], a["bp"], a["ws"], a["wsb"], a["s"])
+
+
+@pytest.mark.parametrize("kw,code", [
+    # the checks of aces_verify ...
+    (dict(B=0), 1), (dict(K=17), 1), (dict(T=0.0), 2), (dict(top_p=0.0), 1), (dict(k=257), 1),
+    (dict(dt=7), 2), (dict(z=None), 1), (dict(u=None), 1), (dict(ws=None), 1), (dict(wsb=16), 1),
+    # ... and those of aces_cache_build, all before any launch
+    (dict(F=None), 1), (dict(F=(ctypes.c_int32 * 4)(2, -1, 2, 2)), 1),
+    (dict(V=5000, F=(ctypes.c_int32 * 4)(2, 2000, 2, 2)), 2), (dict(bt=None), 1), (dict(bp=None), 1),
+])
+def test_cloud_step_rejects_invalid_arguments(lib, kw, code):
+    assert _step(lib, **kw) == code
+
+
 def test_cache_calls_reject_invalid_arguments(lib):
     F = (ctypes.c_int32 * 4)(2, 2, 2, 2)
     Fbad = (ctypes.c_int32 * 4)(2, -1, 2, 2)
