@@ -314,6 +314,8 @@ def main():
     ap.add_argument("--ref-seqs", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the resample and KV-compaction timings (small profiling runs)")
     ap.add_argument("--e2e-steps", type=int, default=0)
     ap.add_argument("--B", type=int, default=0, help="use only the first B sequences (small profiling runs)")
     args = ap.parse_args()
@@ -436,58 +438,59 @@ def main():
                         "gbs": cb / (part_ms["cache_build"] * 1e-3) / 1e9, "kernels": ["k_cache_build"]},
         "cache_lookup": {"ms": part_ms["cache_lookup"], "kernels": ["k_cache_lookup"]},
     }
-    # edge-side draw from the sparse payload (Alg. 1 RESAMPLE), timed apart from the step
-    rs_out = A.resample_sparse(out["accept_len"], out["topk_ids"], out["topk_probs"], out["tail_mass"],
-                               out["row_status"], d["q"], d["u"])
-    for _ in range(3):
-        A.resample_sparse(out["accept_len"], out["topk_ids"], out["topk_probs"], out["tail_mass"],
-                          out["row_status"], d["q"], d["u"], out=rs_out)
-    r0 = torch.cuda.Event(enable_timing=True)
-    r1 = torch.cuda.Event(enable_timing=True)
-    r0.record(stream)
-    for _ in range(args.steps):
-        A.resample_sparse(out["accept_len"], out["topk_ids"], out["topk_probs"], out["tail_mass"],
-                          out["row_status"], d["q"], d["u"], out=rs_out)
-    r1.record(stream)
-    torch.cuda.synchronize()
-    rs_ms = r0.elapsed_time(r1) / args.steps
-    tail_pi = out["tail_mass"][torch.arange(B, device=dev), out["accept_len"].long()].cpu().numpy()
-    n_spread = int((tail_pi > 0).sum())
-    rb = resample_bytes(B, K, V, k, n_spread)
-    parts["resample_sparse"] = {"ms": rs_ms, "alg_bytes": rb, "gbs": rb / (rs_ms * 1e-3) / 1e9,
-                                "sequences_reading_whole_q_row": n_spread, "kernels": ["k_resample_sparse"],
-                                "note": "edge-side draw from row pi's payload; not part of the step"}
-    # COMPACT_KV after the lookup (Alg. 1), timed apart from the step: a draft
-    # model's KV cache (28 layers x {K, V}, 8 heads, head dim 128, bf16) for
-    # the first 64 sequences, prefix of 512 positions, branches of K + 1
-    kb = min(B, 64)
-    planes, kh, kd, t0, bl = 56, 8, 128, 512, K + 1
-    S_kv = t0 + K + S * bl
-    kv = torch.empty(planes, kb, kh, S_kv, kd, dtype=torch.bfloat16, device=dev)
-    pref = torch.full((kb,), t0, dtype=torch.int32, device=dev)
-    new_len = torch.empty(kb, dtype=torch.int32, device=dev)
-    kv_args = (kv, pref, out["accept_len"][:kb], slot[:kb], K, bl)
-    for _ in range(3):
-        A.compact_kv(*kv_args, new_len=new_len)
-    # the moved rows (tens of MB) fit in L2: flush it (write 256 MB) before each timed call
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
-    kv_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-             for _ in range(args.steps)]
-    for e0, e1 in kv_ev:
-        flush.fill_(1)
-        e0.record(stream)
-        A.compact_kv(*kv_args, new_len=new_len)
-        e1.record(stream)
-    torch.cuda.synchronize()
-    kv_ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in kv_ev)
-    del flush
-    n_hit = int((slot[:kb] >= 0).sum().item())
-    kvb = 2 * n_hit * planes * kh * bl * kd * 2
-    parts["compact_kv"] = {"ms": kv_ms, "alg_bytes": kvb, "gbs": kvb / (kv_ms * 1e-3) / 1e9, "hits": n_hit,
-                           "sequences": kb, "kernels": ["k_compact_kv"],
-                           "note": "KV [56, 64, 8, %d, 128] bf16; moved rows read + written; L2 flushed before each "
-                                   "call; not part of the step" % S_kv}
-    del kv
+    if not args.no_extras:
+        # edge-side draw from the sparse payload (Alg. 1 RESAMPLE), timed apart from the step
+        rs_out = A.resample_sparse(out["accept_len"], out["topk_ids"], out["topk_probs"], out["tail_mass"],
+                                   out["row_status"], d["q"], d["u"])
+        for _ in range(3):
+            A.resample_sparse(out["accept_len"], out["topk_ids"], out["topk_probs"], out["tail_mass"],
+                              out["row_status"], d["q"], d["u"], out=rs_out)
+        r0 = torch.cuda.Event(enable_timing=True)
+        r1 = torch.cuda.Event(enable_timing=True)
+        r0.record(stream)
+        for _ in range(args.steps):
+            A.resample_sparse(out["accept_len"], out["topk_ids"], out["topk_probs"], out["tail_mass"],
+                              out["row_status"], d["q"], d["u"], out=rs_out)
+        r1.record(stream)
+        torch.cuda.synchronize()
+        rs_ms = r0.elapsed_time(r1) / args.steps
+        tail_pi = out["tail_mass"][torch.arange(B, device=dev), out["accept_len"].long()].cpu().numpy()
+        n_spread = int((tail_pi > 0).sum())
+        rb = resample_bytes(B, K, V, k, n_spread)
+        parts["resample_sparse"] = {"ms": rs_ms, "alg_bytes": rb, "gbs": rb / (rs_ms * 1e-3) / 1e9,
+                                    "sequences_reading_whole_q_row": n_spread, "kernels": ["k_resample_sparse"],
+                                    "note": "edge-side draw from row pi's payload; not part of the step"}
+        # COMPACT_KV after the lookup (Alg. 1), timed apart from the step: a draft
+        # model's KV cache (28 layers x {K, V}, 8 heads, head dim 128, bf16) for
+        # the first 64 sequences, prefix of 512 positions, branches of K + 1
+        kb = min(B, 64)
+        planes, kh, kd, t0, bl = 56, 8, 128, 512, K + 1
+        S_kv = t0 + K + S * bl
+        kv = torch.empty(planes, kb, kh, S_kv, kd, dtype=torch.bfloat16, device=dev)
+        pref = torch.full((kb,), t0, dtype=torch.int32, device=dev)
+        new_len = torch.empty(kb, dtype=torch.int32, device=dev)
+        kv_args = (kv, pref, out["accept_len"][:kb], slot[:kb], K, bl)
+        for _ in range(3):
+            A.compact_kv(*kv_args, new_len=new_len)
+        # the moved rows (tens of MB) fit in L2: flush it (write 256 MB) before each timed call
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+        kv_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                 for _ in range(args.steps)]
+        for e0, e1 in kv_ev:
+            flush.fill_(1)
+            e0.record(stream)
+            A.compact_kv(*kv_args, new_len=new_len)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        kv_ms = statistics.mean(e0.elapsed_time(e1) for e0, e1 in kv_ev)
+        del flush
+        n_hit = int((slot[:kb] >= 0).sum().item())
+        kvb = 2 * n_hit * planes * kh * bl * kd * 2
+        parts["compact_kv"] = {"ms": kv_ms, "alg_bytes": kvb, "gbs": kvb / (kv_ms * 1e-3) / 1e9, "hits": n_hit,
+                               "sequences": kb, "kernels": ["k_compact_kv"],
+                               "note": "KV [56, 64, 8, %d, 128] bf16; moved rows read + written; L2 flushed before each "
+                                       "call; not part of the step" % S_kv}
+        del kv
     for p in parts.values():
         if "gbs" in p:
             p["frac_of_peak"] = p["gbs"] / peak

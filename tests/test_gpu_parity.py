@@ -141,6 +141,10 @@ RAGGED = [
     dict(B=2, K=4, V=2, dtype="f32", T=1.0, top_p=0.5, k=2),           # smallest vocabulary
     dict(B=3, K=3, V=50000, dtype="bf16", T=0.3, top_p=0.05, k=8, rho=0.95),  # one-id nucleus
     dict(B=2, K=2, V=300000, dtype="bf16", T=0.9, top_p=0.9, k=32, zipf=True),  # larger sketch groups
+    # the largest vocabulary (ACES_MAX_V = 2^20): bf16 rows fill the sketch
+    # exactly (16384 groups of 8 chunks), float32 rows exceed it (general path)
+    dict(B=1, K=1, V=1 << 20, dtype="bf16", T=0.8, top_p=0.9, k=64),
+    dict(B=1, K=1, V=1 << 20, dtype="f32", T=0.8, top_p=0.9, k=64),
 ]
 
 
