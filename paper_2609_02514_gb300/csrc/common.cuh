@@ -366,7 +366,8 @@ struct Workspace {
     int *fb_count;             // [8]   [0] rows handed to the general path, [1] wait timeouts,
                                //       [2] rows certified by the full sketch, [3] rows ordered by
                                //       bitonic sort, [4] rows the general path finished by radix
-                               //       selection, [5] rows split over several CTAs (path
+                               //       selection, [5] rows split over several CTAs, [6] rows
+                               //       the general path finished by value histogram (path
                                //       counters, cleared by every call)
     RowStat *stats;            // [rows]
     int *acc;                  // [B*K] accept bits

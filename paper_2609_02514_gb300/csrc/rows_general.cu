@@ -433,11 +433,214 @@ __device__ bool binned_row(const RowArgs &a, int r, const char *row, float m, fl
     return true;
 }
 
+// ---------------------------------------------------------------------------
+// Value-histogram path for bfloat16 rows.  A bfloat16 logit takes one of
+// 65536 values, and equal values have equal masses, so counting the elements
+// of each value is enough: the VH_W values below the row max get a count
+// (one shared-memory atomic per element, no per-element mass), and the
+// exp-sum S of the whole row is a compensated fp32 sum, as in the fast
+// kernel.  A prefix scan over the values then gives, exactly in 2^-40 fixed
+// point (count x the value's mass), the value holding the nucleus crossing
+// (first prefix reaching ceil(top_p * S * 2^40)) and the value holding the
+// k-th payload id; the elements of those values (ties are taken in id order,
+// which is the order-value order) are collected and ordered in shared
+// memory.  Returns false, having written nothing, when a needed value lies
+// below the window or a collected set exceeds VH_CAP; the binned path then
+// takes the row.
+constexpr int VH_W = 4096;    // values below the max with a count
+constexpr int VH_CAP = 1024;  // collected ids per set (payload values, crossing value)
+
+struct ValHist {
+    uint32_t cnt[VH_W];                // elements of value key16(max) - d
+    unsigned long long pay[VH_CAP];    // order values of the payload values
+    unsigned long long tie[VH_CAP];    // order values of the crossing value
+    int npay, ntie;
+    int dstar, dk, j;                  // crossing value, last payload value, ids of dstar in the nucleus
+    unsigned long long above, cnt_above, npay_need;
+};
+
+// 16-bit order key of a bfloat16 value (the high half of fkey of the value,
+// with -0 taken as +0), and the value of a key
+__device__ __forceinline__ uint32_t bkey16(uint32_t b) {
+    b = b == 0x8000u ? 0u : b;
+    return (b & 0x8000u) ? (~b & 0xFFFFu) : (b | 0x8000u);
+}
+__device__ __forceinline__ float bval16(uint32_t k) {
+    const uint32_t b = (k & 0x8000u) ? (k & 0x7FFFu) : (~k & 0xFFFFu);
+    return __uint_as_float(b << 16);
+}
+
+// appends o to arr[*n] for every lane with take (one atomic per warp); *n
+// may pass cap, entries beyond it are dropped
+__device__ __forceinline__ void warp_append_cap(unsigned long long *arr, int *n, bool take, unsigned long long o,
+                                                int cap) {
+    const unsigned bal = __ballot_sync(0xffffffffu, take);
+    if (bal == 0u) return;
+    const int lane = threadIdx.x & 31;
+    int base = 0;
+    if (lane == __ffs(bal) - 1) base = atomicAdd(n, __popc(bal));
+    base = __shfl_sync(0xffffffffu, base, __ffs(bal) - 1);
+    const int pos = base + __popc(bal & ((1u << lane) - 1u));
+    if (take && pos < cap) arr[pos] = o;
+}
+
+// (aligned bfloat16 rows; all threads of the CTA)
+__device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, float kref, unsigned long long n_fin,
+                            ValHist *vh, unsigned long long *buf, double *redd, unsigned long long *redu) {
+    using E = Elem<ACES_BF16>;
+    const int tid = threadIdx.x, lane = tid & 31;
+    const bool all_in = a.top_p >= 1.0f;
+    const uint32_t km = fkey(m) >> 16;  // m is a bfloat16 value: its 16-bit key
+    for (int i = tid; i < VH_W; i += NT) vh->cnt[i] = 0u;
+    if (tid == 0) {
+        vh->npay = 0;
+        vh->ntie = 0;
+        vh->dstar = all_in ? -1 : -2;  // -2: not (yet) found in the window
+        vh->dk = -2;
+    }
+    __syncthreads();
+    // ---- pass 1: counts per value and the compensated exp-sum ----
+    float hi = 0.f, lo = 0.f;
+    const int nch = a.V / E::EPC;
+    for (int cc = tid; cc < nch; cc += NT) {
+        const uint4 w = ldg16(row + (size_t)cc * 16);
+        const uint32_t wd[4] = {w.x, w.y, w.z, w.w};
+        float cs = 0.f;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const uint32_t b = h ? (wd[q] >> 16) : (wd[q] & 0xFFFFu);
+                cs += ex2(fmaf(__uint_as_float(b << 16), a.c, -kref));  // 0 for -inf
+                const uint32_t d = km - bkey16(b);
+                if (d < (uint32_t)VH_W && b != 0xFF80u) atomicAdd(&vh->cnt[d], 1u);  // (not -inf)
+            }
+        }
+        const float t = hi + cs;  // Neumaier
+        if (fabsf(hi) >= fabsf(cs)) lo += (hi - t) + cs;
+        else lo += (cs - t) + hi;
+        hi = t;
+    }
+    const double S = block_reduce((double)hi + (double)lo, redd, SumD());  // (its barriers order the counts)
+    if (!(S > 0.0 && S < 1e300)) return false;
+    const unsigned long long tg = all_in ? 0ull : (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
+    // ---- prefix scan over the values, PER consecutive values per thread ----
+    constexpr int PER = VH_W / NT;
+    static_assert(VH_W % NT == 0, "whole values per thread");
+    const int d0 = tid * PER;
+    // the mass of the c ids of value km - d (exact: c equal fixed-point masses)
+    auto bin_mass = [&](int d, uint32_t c) -> unsigned long long {
+        return c ? (unsigned long long)c * to_fx(ex2(fmaf(bval16(km - (uint32_t)d), a.c, -kref))) : 0ull;
+    };
+    unsigned long long bm_loc = 0ull, bc_loc = 0ull;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+        const uint32_t c = vh->cnt[d0 + i];
+        bm_loc += bin_mass(d0 + i, c);
+        bc_loc += c;
+    }
+    unsigned long long m_tot, c_tot;
+    const unsigned long long m_ex = block_exscan_n<NT>(bm_loc, redu, &m_tot);
+    const unsigned long long c_ex = block_exscan_n<NT>(bc_loc, redu, &c_tot);
+    if (!all_in) {  // the value whose masses cross tg (at most one thread finds it)
+        unsigned long long cm = m_ex, cc = c_ex;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const uint32_t c = vh->cnt[d0 + i];
+            const unsigned long long bm = bin_mass(d0 + i, c);
+            if (bm > 0ull && cm < tg && cm + bm >= tg) {
+                const unsigned long long e = bm / c;  // one id's mass
+                vh->dstar = d0 + i;
+                vh->above = cm;
+                vh->cnt_above = cc;
+                vh->j = (int)((tg - cm + e - 1) / e);  // ids of this value in the nucleus
+            }
+            cm += bm;
+            cc += c;
+        }
+    }
+    __syncthreads();
+    if (vh->dstar == -2) return false;  // the crossing lies below the window
+    const unsigned long long n_nuc = all_in ? n_fin : vh->cnt_above + (unsigned long long)vh->j;
+    const int L = (int)(n_nuc < (unsigned long long)a.k ? n_nuc : (unsigned long long)a.k);
+    if (L > 0) {  // the value holding the L-th id (at most one thread finds it)
+        unsigned long long cc = c_ex;
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+            const unsigned long long c = vh->cnt[d0 + i];
+            if (cc < (unsigned long long)L && cc + c >= (unsigned long long)L) {
+                vh->dk = d0 + i;
+                vh->npay_need = cc + c;  // ids of the values up to it
+            }
+            cc += c;
+        }
+    } else if (tid == 0) {
+        vh->dk = -1;  // no payload
+    }
+    __syncthreads();
+    const int dstar = vh->dstar, dk = vh->dk;
+    if (dk == -2) return false;  // the L-th id lies below the window
+    if (dk >= 0 && vh->npay_need > (unsigned long long)VH_CAP) return false;
+    if (dstar >= 0 && vh->cnt[dstar] > (uint32_t)VH_CAP) return false;
+    // ---- collect every id of the values up to dk, and those of dstar ----
+    for (int c0 = tid & ~31; c0 < nch; c0 += NT) {  // warp-uniform rounds
+        const int c = c0 + lane;
+        const bool in = c < nch;
+        const uint4 w = in ? ldg16(row + (size_t)c * 16) : make_uint4(0u, 0u, 0u, 0u);
+        const uint32_t wd[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const uint32_t b = h ? (wd[q] >> 16) : (wd[q] & 0xFFFFu);
+                const uint32_t d = km - bkey16(b);
+                const bool fin = in && b != 0xFF80u;
+                const bool tp = fin && dk >= 0 && d <= (uint32_t)dk;
+                const bool tt = fin && dstar >= 0 && d == (uint32_t)dstar;
+                if (!__any_sync(0xffffffffu, tp || tt)) continue;
+                const unsigned long long o =
+                    order_val(fkey(__uint_as_float(b << 16)), (uint32_t)(c * E::EPC + 2 * q + h));
+                warp_append_cap(vh->pay, &vh->npay, tp, o, VH_CAP);
+                warp_append_cap(vh->tie, &vh->ntie, tt, o, VH_CAP);
+            }
+        }
+    }
+    __syncthreads();
+    const int npay = vh->npay, ntie = vh->ntie;
+    // ---- order both sets (descending order value: ties by ascending id) ----
+    {
+        const int p2 = next_pow2(npay < 2 ? 2 : npay), t2 = next_pow2(ntie < 2 ? 2 : ntie);
+        for (int i = npay + tid; i < p2; i += NT) vh->pay[i] = 0ull;
+        for (int i = ntie + tid; i < t2; i += NT) vh->tie[i] = 0ull;
+        __syncthreads();
+        if (dk >= 0) bitonic_sort_desc(vh->pay, p2);
+        if (dstar >= 0) bitonic_sort_desc(vh->tie, t2);
+    }
+    double S_nuc = S;
+    unsigned long long cut = 0ull;
+    if (dstar >= 0) {
+        const int j = vh->j;
+        cut = vh->tie[j - 1];
+        const unsigned long long ed = to_fx(ex2(fmaf(bval16(km - (uint32_t)dstar), a.c, -kref)));
+        S_nuc = (double)(vh->above + (unsigned long long)j * ed) * FX_INV;
+    }
+    const int LL = L < npay ? L : npay;
+    for (int i = tid; i < LL; i += NT) buf[i] = vh->pay[i];
+    __syncthreads();
+    if (tid == 0) atomicAdd(&a.ws.fb_count[6], 1);
+    finish_row<ACES_BF16>(a, r, row, kref, S_nuc, cut, all_in ? RS_ALL_IN : 0, buf, LL, redd);
+    return true;
+}
+
 template <int DT, bool VEC>
 __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
     using E = Elem<DT>;
     __shared__ SelState st;
-    __shared__ BinState bst;
+    __shared__ union {
+        BinState bs;   // binned path
+        ValHist vh;    // value-histogram path (bfloat16)
+    } paths;
+    BinState &bst = paths.bs;
     __shared__ unsigned long long buf[ACES_MAX_TOPK];
     __shared__ double redd[NWARP];
     __shared__ float redf[NWARP];
@@ -470,6 +673,11 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
             __syncthreads();
             continue;
         }
+        if (DT == ACES_BF16 && VEC && valhist_row(a, r, row, m, kref, n_fin, &paths.vh, buf, redd, redu)) {
+            __syncthreads();
+            continue;
+        }
+        __syncthreads();  // the value histogram shares its memory with the binned path
         if (binned_row<DT, VEC>(a, r, row, m, kref, n_fin, &bst, buf, redd, redu)) {
             __syncthreads();
             continue;

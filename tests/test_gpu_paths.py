@@ -4,8 +4,8 @@ The workspace's first int32 words count, per call, the rows handed to the
 exact general kernel, bounded-wait timeouts, rows certified only by the full
 sketch histogram (the top group maxima kept per thread were not enough),
 rows whose candidates were ordered by bitonic sort (more than 512), rows the
-general kernel finished by radix selection, and rows split over several
-CTAs.  Each
+general kernel finished by radix selection, rows split over several CTAs,
+and rows the general kernel finished by its bfloat16 value histogram.  Each
 test asserts the branch it targets was taken, then compares every output
 with the float64 oracle under the rules of tests/parity.py.
 """
@@ -44,7 +44,7 @@ def _run(A, orc, w, z):
     g = A.verify(zt, q, xt, u, w.T, w.top_p, w.k, workspace=ws)
     torch.cuda.synchronize()
     g = {key: v.cpu().numpy() for key, v in g.items()}
-    counters = ws[:24].view(torch.int32).cpu().numpy().tolist()
+    counters = ws[:28].view(torch.int32).cpu().numpy().tolist()
     o = orc.verify(z, inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
     res = parity.compare_verify(inp, g, o, w.top_p, z.dtype == np.uint16, w.k)
     return counters, res
@@ -68,7 +68,7 @@ def test_second_tier_certification_and_bitonic_order(A, orc):
     # sketch certifies, and the nucleus (~1200 ids) is ordered by bitonic sort
     w = gen.make_workload(2, 2, 32000, "f32", T=1.0, top_p=0.8, k=64, seed=31)
     counters, res = _run(A, orc, w, _plateau(2, 2, 32000, 1500, 16, 31))
-    fallback, timeouts, second_tier, bitonic, radix, split = counters
+    fallback, timeouts, second_tier, bitonic, radix, split, valhist = counters
     assert fallback == 0 and timeouts == 0
     # a row split over CTAs bins every part's top maxima, which here covers
     # every hot group: the first tier then suffices
@@ -108,3 +108,65 @@ def test_large_vocabularies(A, orc, dtype, V):
     counters, res = _run(A, orc, w, z)
     assert counters[1] == 0
     assert res["checked_seqs"] == 1
+
+
+def _bf16(z):
+    return gen.f32_to_bf16(np.ascontiguousarray(z, dtype=np.float32))
+
+
+def test_value_histogram_takes_large_nucleus_bf16_rows(A, orc):
+    # rows of the 128256-id recipe (nuclei of thousands of ids): the sketch
+    # cannot order them, and the general kernel finishes every one by counting
+    # ids per bf16 value (the crossing lies among the 4096 values below the max)
+    w = gen.make_workload(2, 2, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=41)
+    z = gen.generate(w)["z"]
+    counters, res = _run(A, orc, w, z)
+    fallback, radix, valhist = counters[0], counters[4], counters[6]
+    assert fallback >= 1 and valhist == fallback and radix == 0, counters
+    assert res["checked_seqs"] >= 1
+
+
+def test_value_histogram_declines_a_crossing_below_its_window(A, orc):
+    # flat rows (T=2, top_p=0.99): the crossing lies among negative logits,
+    # whose keys are below the window (below every tiny positive value); the
+    # binned path takes the rows
+    w = gen.make_workload(3, 2, 65536, "bf16", T=2.0, top_p=0.99, k=64, seed=41)
+    z = gen.generate(w)["z"]
+    counters, res = _run(A, orc, w, z)  # (compares every unflagged output)
+    fallback, valhist = counters[0], counters[6]
+    assert fallback >= 1 and valhist == 0, counters
+
+
+@pytest.mark.parametrize("n_vals,V,expect_valhist", [(40, 32000, True), (24, 65536, False)],
+                         ids=["ties_within_capacity", "ties_beyond_capacity"])
+def test_value_histogram_ties(A, orc, n_vals, V, expect_valhist):
+    # logits from a few distinct bf16 values: the crossing value is shared by
+    # ~V/n_vals ids, taken in id order.  Up to 1024 of them the value
+    # histogram orders them itself; beyond that the binned path takes the row.
+    w = gen.make_workload(2, 2, V, "bf16", T=1.0, top_p=0.7, k=32, seed=42)
+    rng = np.random.default_rng(42)
+    vals = np.linspace(-2.0, 2.0, n_vals).astype(np.float32)
+    z = _bf16(vals[rng.integers(0, n_vals, size=(2, 3, V))])
+    counters, res = _run(A, orc, w, z)
+    fallback, valhist = counters[0], counters[6]
+    assert fallback == 6, counters
+    assert (valhist == 6) if expect_valhist else (valhist == 0), counters
+    assert res["checked_seqs"] >= 1
+
+
+def test_signed_zeros_on_the_general_path(A, orc):
+    # -0 and +0 are one value (one order key): the nucleus and the payload take
+    # them in id order whatever their signs.  Ten positive ids, then a run of
+    # 512 zeros of random sign (16 whole sketch groups, so the one-max-per-group
+    # bound cannot certify the row), the rest at -20.  Zero lies ~16000 bf16
+    # keys below a max near 1, beyond the value histogram's window, so the
+    # binned path takes the rows.
+    V = 32000
+    w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.999, k=64, seed=43)
+    rng = np.random.default_rng(43)
+    z = np.full((2, 2, V), -20.0, np.float32)
+    z[:, :, 100:110] = rng.uniform(0.5, 1.0, size=(2, 2, 10)).astype(np.float32)
+    z[:, :, 1024:1536] = np.where(rng.random((2, 2, 512)) < 0.5, np.float32(0.0), np.float32(-0.0))
+    counters, res = _run(A, orc, w, _bf16(z))
+    assert counters[0] == 4 and counters[6] == 0, counters
+    assert res["checked_seqs"] >= 1
