@@ -17,6 +17,7 @@ constexpr int BIN_PER_T = 8;
 // Row-level flags kept in the workspace.
 constexpr int RS_ALL_IN = 1;        // top_p >= 1: every finite id is in the nucleus
 constexpr int RS_NONFINITE = 2;
+constexpr int RS_HANDOFF = 4;       // handed to the general kernel; kref holds the row max
 
 // Per-row state written by the row kernels and read by the resolve kernel.
 struct RowStat {

@@ -485,8 +485,11 @@ __device__ __forceinline__ void warp_append_cap(unsigned long long *arr, int *n,
 }
 
 // (aligned bfloat16 rows; all threads of the CTA)
-__device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, float kref, unsigned long long n_fin,
-                            ValHist *vh, unsigned long long *buf, double *redd, unsigned long long *redu) {
+// *n_fin_out gets the row's count of finite ids (computed by pass 1) even
+// when the row is declined.
+__device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, float kref,
+                            unsigned long long *n_fin_out, ValHist *vh, unsigned long long *buf, double *redd,
+                            unsigned long long *redu) {
     using E = Elem<ACES_BF16>;
     const int tid = threadIdx.x, lane = tid & 31;
     const bool all_in = a.top_p >= 1.0f;
@@ -501,6 +504,7 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
     __syncthreads();
     // ---- pass 1: counts per value and the compensated exp-sum ----
     float hi = 0.f, lo = 0.f;
+    unsigned long long nfin = 0ull;
     const int nch = a.V / E::EPC;
     for (int cc = tid; cc < nch; cc += NT) {
         const uint4 w = ldg16(row + (size_t)cc * 16);
@@ -512,8 +516,10 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
             for (int h = 0; h < 2; ++h) {
                 const uint32_t b = h ? (wd[q] >> 16) : (wd[q] & 0xFFFFu);
                 cs += ex2(fmaf(__uint_as_float(b << 16), a.c, -kref));  // 0 for -inf
+                const bool fin = b != 0xFF80u;
+                nfin += fin;
                 const uint32_t d = km - bkey16(b);
-                if (d < (uint32_t)VH_W && b != 0xFF80u) atomicAdd(&vh->cnt[d], 1u);  // (not -inf)
+                if (d < (uint32_t)VH_W && fin) atomicAdd(&vh->cnt[d], 1u);
             }
         }
         const float t = hi + cs;  // Neumaier
@@ -521,6 +527,8 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
         else lo += (cs - t) + hi;
         hi = t;
     }
+    const unsigned long long n_fin = block_reduce(nfin, redu, SumU64());
+    *n_fin_out = n_fin;
     const double S = block_reduce((double)hi + (double)lo, redd, SumD());  // (its barriers order the counts)
     if (!(S > 0.0 && S < 1e300)) return false;
     const unsigned long long tg = all_in ? 0ull : (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
@@ -653,31 +661,41 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
     for (int idx = blockIdx.x; idx < nrows; idx += gridDim.x) {
         const int r = direct ? idx : a.ws.fb_list[idx];
         const char *row = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
-        // pass 0: max, finite count, invalid values
-        if (tid == 0) s_bad = 0;
-        __syncthreads();
-        float mx = -INFINITY;
-        unsigned long long nfin = 0;
-        int bad = 0;
-        for_each_elem<DT, VEC>(row, a.V, [&](int, float v) {
-            if (v != v || v == INFINITY) bad = 1;
-            if (v > -INFINITY) ++nfin;
-            mx = fmaxf(mx, v);
-        });
-        if (bad) s_bad = 1;
-        const float m = block_reduce(mx, redf, MaxF());
+        // a row the fast kernel handed over comes with its max (and is finite)
+        const bool handed = DT == ACES_BF16 && VEC && !direct && a.ws.stats[r].flags == RS_HANDOFF;
+        float m;
+        unsigned long long n_fin = 0ull;
+        if (handed) {
+            m = a.ws.stats[r].kref;
+        } else {
+            // pass 0: max, finite count, invalid values
+            if (tid == 0) s_bad = 0;
+            __syncthreads();
+            float mx = -INFINITY;
+            unsigned long long nfin = 0;
+            int bad = 0;
+            for_each_elem<DT, VEC>(row, a.V, [&](int, float v) {
+                if (v != v || v == INFINITY) bad = 1;
+                if (v > -INFINITY) ++nfin;
+                mx = fmaxf(mx, v);
+            });
+            if (bad) s_bad = 1;
+            m = block_reduce(mx, redf, MaxF());
+            n_fin = block_reduce(nfin, redu, SumU64());
+            if (s_bad || n_fin == 0ull || !(ceilf(m * a.c) < 1e30f)) {
+                nonfinite_row<NT>(a, r);
+                __syncthreads();
+                continue;
+            }
+        }
         const float kref = ceilf(m * a.c);  // masses are 2^(z*c - kref) <= 1
-        const unsigned long long n_fin = block_reduce(nfin, redu, SumU64());
-        if (s_bad || n_fin == 0ull || !(kref < 1e30f)) {
-            nonfinite_row<NT>(a, r);
+        if (DT == ACES_BF16 && VEC) {
+            unsigned long long nf = 0ull;
+            const bool done = valhist_row(a, r, row, m, kref, &nf, &paths.vh, buf, redd, redu);
             __syncthreads();
-            continue;
+            if (done) continue;
+            n_fin = nf;
         }
-        if (DT == ACES_BF16 && VEC && valhist_row(a, r, row, m, kref, n_fin, &paths.vh, buf, redd, redu)) {
-            __syncthreads();
-            continue;
-        }
-        __syncthreads();  // the value histogram shares its memory with the binned path
         if (binned_row<DT, VEC>(a, r, row, m, kref, n_fin, &bst, buf, redd, redu)) {
             __syncthreads();
             continue;
