@@ -66,8 +66,8 @@ typedef enum { ACES_F32 = 0, ACES_BF16 = 1 } aces_dtype;
 /* bits of row_status */
 #define ACES_ROW_NONFINITE 1 /* NaN / +inf logits, or all logits -inf      */
 #define ACES_ROW_BAD_Q 2     /* invalid draft probability or draft token   */
-#define ACES_ROW_TIMEOUT 4   /* a bounded wait inside a kernel gave up; the
-                                row's outputs are padding (never expected) */
+#define ACES_ROW_TIMEOUT 4   /* reserved for a kernel that gives up a bounded
+                                wait; no current kernel waits on another */
 
 /* The CUDA runtime's cudaStream_t (NULL = legacy default stream). */
 typedef struct CUstream_st *aces_stream_t;

@@ -294,63 +294,6 @@ __device__ __forceinline__ unsigned long long floor_u_times(float uu, unsigned l
     return thr;
 }
 
-// ---------------------------------------------------------------------------
-// mbarrier and bulk async copy (global -> shared), CTA scope
-__device__ __forceinline__ uint32_t smem_u32(const void *p) {
-    return (uint32_t)__cvta_generic_to_shared(p);
-}
-__device__ __forceinline__ void mbar_init(unsigned long long *bar, unsigned count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_fence_init() {
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(unsigned long long *bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-                 : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(unsigned long long *bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(unsigned long long *bar, uint32_t phase) {
-    uint32_t done;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(done)
-        : "r"(smem_u32(bar)), "r"(phase)
-        : "memory");
-    return done != 0u;
-}
-// Waits for the phase with the given parity to complete; gives up after
-// about one second (2^31 SM clock cycles) and returns false.
-__device__ __forceinline__ bool mbar_wait_bounded(unsigned long long *bar, uint32_t phase) {
-    if (mbar_try_wait(bar, phase)) return true;
-    const long long t0 = clock64();
-    while (!mbar_try_wait(bar, phase)) {
-        if (clock64() - t0 > (1ll << 31)) return false;
-    }
-    return true;
-}
-// per-thread async copy of 16 bytes, global -> shared (both 16-byte aligned)
-__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-// bytes and both addresses must be multiples of 16
-__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, unsigned long long *bar) {
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-            smem_u32(dst)),
-        "l"(src), "r"(bytes), "r"(smem_u32(bar))
-        : "memory");
-}
-
 // Exact sums of one vocabulary segment of a sequence's row pi (2^-40 units).
 struct SegSum {
     unsigned long long r;  // residual max(0, p - q)
@@ -364,7 +307,8 @@ constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual s
 constexpr int WS_COUNTERS = 32;  // bytes of path counters at the start of the workspace
 // Workspace layout (all offsets 16-byte aligned)
 struct Workspace {
-    int *fb_count;             // [8]   [0] rows handed to the general path, [1] wait timeouts,
+    int *fb_count;             // [8]   [0] rows handed to the general path, [1] reserved (no
+                               //       kernel waits on another),
                                //       [2] rows certified by the full sketch, [3] rows ordered by
                                //       bitonic sort, [4] rows the general path finished by radix
                                //       selection, [5] rows split over several CTAs, [6] rows
@@ -641,14 +585,6 @@ __device__ void nonfinite_row(const RowArgs &a, int r) {
         s.nnuc = -1;
         a.ws.stats[r] = s;
     }
-}
-
-// Outputs of a row whose kernel gave up on a wait (never expected).
-template <int NTH>
-__device__ void timeout_row(const RowArgs &a, int r) {
-    nonfinite_row<NTH>(a, r);
-    __syncthreads();
-    if (threadIdx.x == 0) a.row_status[r] = ACES_ROW_TIMEOUT;
 }
 
 // host launchers (defined next to their kernels)
