@@ -14,10 +14,13 @@
  *
  * Conventions shared by every entry point
  *   - All array arguments are DEVICE pointers owned by the caller; the
- *     library never allocates, frees or retains them.  F_host is the one
- *     host array.
- *   - Work is enqueued on `stream` and the call returns before it finishes.
- *     A call returns ACES_OK once its kernels are launched.
+ *     library never allocates, frees or retains them, and allocates no
+ *     device memory of its own (aces_cloud_step creates one stream and two
+ *     events per device on its first call there).  F_host is the one host
+ *     array.
+ *   - Work is enqueued on `stream` (aces_cloud_step also on its own stream,
+ *     forked from and joined back to `stream`) and the call returns before
+ *     it finishes.  A call returns ACES_OK once its kernels are launched.
  *   - Arguments are validated before anything is launched; on
  *     ACES_ERR_INVALID_ARG / ACES_ERR_UNSUPPORTED nothing is enqueued and no
  *     output is touched.  ACES_ERR_CUDA reports a failed launch.
