@@ -13,6 +13,8 @@
 //                O = key(z) << 32 | (2^32 - 1 - id), 8 bits per pass.
 #include <climits>
 
+#include <cuda_bf16.h>
+
 #include "common.cuh"
 
 namespace aces {
@@ -591,11 +593,23 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
     if (dk >= 0 && vh->npay_need > (unsigned long long)VH_CAP) return false;
     if (dstar >= 0 && vh->cnt[dstar] > (uint32_t)VH_CAP) return false;
     // ---- collect every id of the values up to dk, and those of dstar ----
+    // (an id is taken only if its value reaches that of key km - max(dk,
+    // dstar): a chunk whose max is below it is skipped with one vote)
+    const float vthr = bval16(km - (uint32_t)(dk > dstar ? dk : dstar));
     for (int c0 = tid & ~31; c0 < nch; c0 += NT) {  // warp-uniform rounds
         const int c = c0 + lane;
         const bool in = c < nch;
-        const uint4 w = in ? ldg16(row + (size_t)c * 16) : make_uint4(0u, 0u, 0u, 0u);
+        const uint4 w = in ? ldg16(row + (size_t)c * 16) : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
         const uint32_t wd[4] = {w.x, w.y, w.z, w.w};
+        {
+            const __nv_bfloat162 m2 = __hmax2(__hmax2(*reinterpret_cast<const __nv_bfloat162 *>(&wd[0]),
+                                                      *reinterpret_cast<const __nv_bfloat162 *>(&wd[1])),
+                                              __hmax2(*reinterpret_cast<const __nv_bfloat162 *>(&wd[2]),
+                                                      *reinterpret_cast<const __nv_bfloat162 *>(&wd[3])));
+            const uint32_t mu = *reinterpret_cast<const uint32_t *>(&m2);
+            const float cmax = fmaxf(__uint_as_float(mu << 16), __uint_as_float(mu & 0xFFFF0000u));
+            if (!__any_sync(0xffffffffu, in && cmax >= vthr)) continue;
+        }
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
 #pragma unroll
