@@ -473,14 +473,15 @@ struct DrawShared {
 // nucleus ids only, which are ordered by id, and the token is the smallest id
 // whose prefix sum of 2^-40 fixed-point masses exceeds floor(u * total).
 // Writes accept_len, out_token and seqdone; returns without writing when row
-// pi has no stored nucleus (the scan kernels then draw the sequence).  All
-// NTH threads call it, NTH * 2 >= NUC_CAP; skey, rfx, pfx hold NUC_CAP
-// entries, red NTH / 32.
+// pi has no stored nucleus (the scan kernels then draw the sequence).  The
+// ids are ordered by direct rank counting (one pass, no barrier stages).
+// All NTH threads call it, NTH * 2 >= NUC_CAP; skey, srt, rfx, pfx hold
+// NUC_CAP entries, red NTH / 32.
 template <int NTH>
 __device__ void draw_from_list(const Workspace &ws, const float *q, const float *u, int K, int V, int b,
                                int32_t *accept_len, int32_t *out_token, int32_t *row_status,
-                               unsigned long long *skey, unsigned long long *rfx, unsigned long long *pfx,
-                               unsigned long long *red, DrawShared *sh) {
+                               unsigned long long *skey, unsigned long long *srt, unsigned long long *rfx,
+                               unsigned long long *pfx, unsigned long long *red, DrawShared *sh) {
     static_assert(2 * NTH >= NUC_CAP, "two nucleus entries per thread");
     const int tid = threadIdx.x;
     if (tid == 0) {
@@ -505,24 +506,19 @@ __device__ void draw_from_list(const Workspace &ws, const float *q, const float 
     const unsigned long long *lst = ws.nuc + (size_t)r * NUC_CAP;
     const float *qrow = pi < K ? q + ((size_t)b * K + pi) * V : nullptr;
     const float inv_S = inv_mass(rs.S_nuc);
-    const int np = next_pow2(n < 2 ? 2 : n);
-    for (int i = tid; i < np; i += NTH) {
-        if (i < n) {
-            const unsigned long long o = lst[i];
-            const uint32_t id = order_id(o);
-            const float p = ex2(fmaf(order_value(o), rs.c, -rs.kref)) * inv_S;
-            float rr = p;
-            if (qrow) {
-                const float qx = __ldg(qrow + id);
-                if (!(qx >= 0.0f)) sh->bad = 1;
-                rr = fmaxf(p - qx, 0.0f);
-            }
-            rfx[i] = to_fx(rr);
-            pfx[i] = to_fx(p);
-            skey[i] = ~(((unsigned long long)id << 32) | (unsigned long long)i);
-        } else {
-            skey[i] = 0ull;
+    for (int i = tid; i < n; i += NTH) {
+        const unsigned long long o = lst[i];
+        const uint32_t id = order_id(o);
+        const float p = ex2(fmaf(order_value(o), rs.c, -rs.kref)) * inv_S;
+        float rr = p;
+        if (qrow) {
+            const float qx = __ldg(qrow + id);
+            if (!(qx >= 0.0f)) sh->bad = 1;
+            rr = fmaxf(p - qx, 0.0f);
         }
+        rfx[i] = to_fx(rr);
+        pfx[i] = to_fx(p);
+        skey[i] = ((unsigned long long)id << 32) | (unsigned long long)i;  // distinct keys
     }
     __syncthreads();
     if (sh->bad) {
@@ -534,11 +530,18 @@ __device__ void draw_from_list(const Workspace &ws, const float *q, const float 
         }
         return;
     }
-    bitonic_sort_desc(skey, np);  // ascending id
+    for (int i = tid; i < n; i += NTH) {  // ascending id: each key's rank among the others
+        const unsigned long long key = skey[i];
+        int rank = 0;
+#pragma unroll 4
+        for (int j = 0; j < n; ++j) rank += skey[j] < key;
+        srt[rank] = key;
+    }
+    __syncthreads();
     // two consecutive entries (in id order) per thread
     const int e0 = 2 * tid, e1 = 2 * tid + 1;
-    const int i0 = e0 < n ? (int)(~skey[e0] & 0xFFFFFFFFull) : -1;
-    const int i1 = e1 < n ? (int)(~skey[e1] & 0xFFFFFFFFull) : -1;
+    const int i0 = e0 < n ? (int)(srt[e0] & 0xFFFFFFFFull) : -1;
+    const int i1 = e1 < n ? (int)(srt[e1] & 0xFFFFFFFFull) : -1;
     const unsigned long long r0 = i0 >= 0 ? rfx[i0] : 0ull, r1 = i1 >= 0 ? rfx[i1] : 0ull;
     const unsigned long long R = block_reduce_n<NTH>(r0 + r1, red, SumU64());
     const int mode = R == 0ull;  // p <= q everywhere: draw from p itself
@@ -550,8 +553,8 @@ __device__ void draw_from_list(const Workspace &ws, const float *q, const float 
     __syncthreads();
     const unsigned long long thr = sh->thr;
     if (tot > 0ull) {
-        if (ex <= thr && thr < ex + w0) sh->tok = (int)(~skey[e0] >> 32);
-        else if (ex + w0 <= thr && thr < ex + w0 + w1) sh->tok = (int)(~skey[e1] >> 32);
+        if (ex <= thr && thr < ex + w0) sh->tok = (int)(srt[e0] >> 32);
+        else if (ex + w0 <= thr && thr < ex + w0 + w1) sh->tok = (int)(srt[e1] >> 32);
     }
     __syncthreads();
     if (tid == 0) {

@@ -162,9 +162,9 @@ __device__ void row_finished(const RowArgs &a, int r, unsigned char *scratch) {
     if (threadIdx.x == 0) s_last = atomic_add_acq_rel(&a.ws.seqcnt[b], 1) == a.K;
     __syncthreads();
     if (!s_last) return;
-    unsigned long long *skey = reinterpret_cast<unsigned long long *>(scratch);
+    unsigned long long *skey = reinterpret_cast<unsigned long long *>(scratch);  // 4 * NUC_CAP entries
     draw_from_list<NTH>(a.ws, a.q, a.u, a.K, a.V, b, a.accept_len, a.out_token, a.row_status, skey,
-                        skey + NUC_CAP, skey + 2 * NUC_CAP, s_red, &s_draw);
+                        skey + NUC_CAP, skey + 2 * NUC_CAP, skey + 3 * NUC_CAP, s_red, &s_draw);
 }
 
 // Hands row r to the general kernel with its max m (the row is finite: rows
