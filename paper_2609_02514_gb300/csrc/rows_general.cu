@@ -459,6 +459,7 @@ struct ValHist {
     int npay, ntie;
     int dstar, dk, j;                  // crossing value, last payload value, ids of dstar in the nucleus
     unsigned long long above, cnt_above, npay_need;
+    unsigned long long above_cut;      // the cut: order value of the crossing value's j-th id
 };
 
 // 16-bit order key of a bfloat16 value (the high half of fkey of the value,
@@ -629,26 +630,33 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
     }
     __syncthreads();
     const int npay = vh->npay, ntie = vh->ntie;
-    // ---- order both sets (descending order value: ties by ascending id) ----
-    {
-        const int p2 = next_pow2(npay < 2 ? 2 : npay), t2 = next_pow2(ntie < 2 ? 2 : ntie);
-        for (int i = npay + tid; i < p2; i += NT) vh->pay[i] = 0ull;
-        for (int i = ntie + tid; i < t2; i += NT) vh->tie[i] = 0ull;
-        __syncthreads();
-        if (dk >= 0) bitonic_sort_desc(vh->pay, p2);
-        if (dstar >= 0) bitonic_sort_desc(vh->tie, t2);
+    // ---- rank by direct counting (order values are distinct; descending
+    // order, ties by ascending id): the first L payload ids go straight to
+    // buf, and the cut is the crossing value's id of rank j - 1 ----
+    const int LL = L < npay ? L : npay;
+    for (int i = tid; i < npay; i += NT) {
+        const unsigned long long key = vh->pay[i];
+        int rank = 0;
+#pragma unroll 4
+        for (int t = 0; t < npay; ++t) rank += vh->pay[t] > key;
+        if (rank < LL) buf[rank] = key;
     }
+    const int jt = dstar >= 0 ? vh->j - 1 : -1;
+    for (int i = tid; i < ntie; i += NT) {
+        const unsigned long long key = vh->tie[i];
+        int rank = 0;
+#pragma unroll 4
+        for (int t = 0; t < ntie; ++t) rank += vh->tie[t] > key;
+        if (rank == jt) vh->above_cut = key;
+    }
+    __syncthreads();
     double S_nuc = S;
     unsigned long long cut = 0ull;
     if (dstar >= 0) {
-        const int j = vh->j;
-        cut = vh->tie[j - 1];
+        cut = vh->above_cut;
         const unsigned long long ed = to_fx(ex2(fmaf(bval16(km - (uint32_t)dstar), a.c, -kref)));
-        S_nuc = (double)(vh->above + (unsigned long long)j * ed) * FX_INV;
+        S_nuc = (double)(vh->above + (unsigned long long)vh->j * ed) * FX_INV;
     }
-    const int LL = L < npay ? L : npay;
-    for (int i = tid; i < LL; i += NT) buf[i] = vh->pay[i];
-    __syncthreads();
     if (tid == 0) atomicAdd(&a.ws.fb_count[6], 1);
     finish_row<ACES_BF16>(a, r, row, kref, S_nuc, cut, all_in ? RS_ALL_IN : 0, buf, LL, redd);
     return true;
