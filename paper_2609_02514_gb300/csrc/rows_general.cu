@@ -389,47 +389,65 @@ __device__ bool binned_row(const RowArgs &a, int r, const char *row, float m, fl
     });
     __syncthreads();
     const int nx = bs->nx, npl = bs->np_;
-    // order both sets (descending order value)
+    // the payload bins' ids ranked by direct counting (order values are
+    // distinct): the first min(npl, k) ranks go straight to buf
+    const int lp = npl < a.k ? npl : a.k;
+    for (int i = tid; i < npl; i += NT) {
+        const unsigned long long key = bs->ps[i];
+        int rank = 0;
+#pragma unroll 4
+        for (int t = 0; t < npl; ++t) rank += bs->ps[t] > key;
+        if (rank < lp) buf[rank] = key;
+    }
+    // the crossing bin in order (descending order value)
     {
         const int p2 = next_pow2(nx < 2 ? 2 : nx);
         for (int i = nx + tid; i < p2; i += NT) bs->xs[i] = 0ull;
-        const int q2 = next_pow2(npl < 2 ? 2 : npl);
-        for (int i = npl + tid; i < q2; i += NT) bs->ps[i] = 0ull;
         __syncthreads();
         if (bx >= 0) bitonic_sort_desc(bs->xs, p2);
-        if (bk >= 0) bitonic_sort_desc(bs->ps, q2);
     }
-    // the crossing id: first id of the crossing bin where the cumulative mass reaches the target
+    // the crossing id: the first id of the crossing bin where the cumulative
+    // mass reaches the target (the bin's last id if rounding keeps it short);
+    // its masses go to ps (free now) and a block scan finds it
     double S_nuc;
     unsigned long long cut = 0ull;
     long long n_nuc;
     if (bx >= 0) {
-        if (tid == 0) {
-            unsigned long long cum = bs->above;
-            int i = 0;
-            for (; i < nx; ++i) {
-                const unsigned long long mi = to_fx(ex2(fmaf(order_value(bs->xs[i]), a.c, -kref)));
-                if ((double)(cum + mi) >= bs->target) {
-                    cum += mi;
-                    break;
-                }
-                cum += mi;
+        for (int i = tid; i < nx; i += NT) bs->ps[i] = to_fx(ex2(fmaf(order_value(bs->xs[i]), a.c, -kref)));
+        if (tid == 0) bs->bk = -1;  // reuse: the crossing position, -1 until found
+        __syncthreads();
+        const int per = (nx + NT - 1) / NT;
+        const int lo = tid * per < nx ? tid * per : nx, hi = lo + per < nx ? lo + per : nx;
+        unsigned long long loc = 0ull;
+        for (int i = lo; i < hi; ++i) loc += bs->ps[i];
+        unsigned long long tot;
+        unsigned long long cum = bs->above + block_exscan_n<NT>(loc, redu, &tot);
+        for (int i = lo; i < hi; ++i) {
+            const unsigned long long prev = cum;
+            cum += bs->ps[i];
+            if ((double)prev < bs->target && (double)cum >= bs->target) {  // one id crosses
+                bs->bk = i;
+                redd[0] = (double)cum * FX_INV;
             }
-            if (i == nx) i = nx - 1;  // rounding: the bin's last id
-            redd[0] = (double)cum * FX_INV;
-            bs->nx = i;  // reuse: position of the crossing in the bin
         }
         __syncthreads();
-        S_nuc = redd[0];
-        cut = bs->xs[bs->nx];
-        n_nuc = (long long)bs->nbelow + bs->nx + 1;
+        int ix = bs->bk;
+        if (ix < 0) {  // rounding: the bin's last id
+            ix = nx - 1;
+            if (tid == 0) redd[1] = (double)(bs->above + tot) * FX_INV;
+            __syncthreads();
+            S_nuc = redd[1];
+        } else {
+            S_nuc = redd[0];
+        }
+        cut = bs->xs[ix];
+        n_nuc = (long long)bs->nbelow + ix + 1;
     } else {
         S_nuc = (double)bs->S_fx * FX_INV;
         n_nuc = (long long)n_fin;
     }
     int L = (int)(n_nuc < (long long)a.k ? n_nuc : (long long)a.k);
-    if (L > npl) L = npl;
-    for (int i = tid; i < L; i += NT) buf[i] = bs->ps[i];
+    if (L > lp) L = lp;
     __syncthreads();
     finish_row<DT>(a, r, row, kref, S_nuc, cut, all_in ? RS_ALL_IN : 0, buf, L, redd);
     return true;
