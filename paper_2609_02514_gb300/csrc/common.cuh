@@ -17,7 +17,9 @@ constexpr int BIN_PER_T = 8;
 // Row-level flags kept in the workspace.
 constexpr int RS_ALL_IN = 1;        // top_p >= 1: every finite id is in the nucleus
 constexpr int RS_NONFINITE = 2;
-constexpr int RS_HANDOFF = 4;       // handed to the general kernel; kref holds the row max
+// handed to the general kernel: kref holds the row max, c the log2 reference
+// of the row's exp-sum and S_nuc that exp-sum
+constexpr int RS_HANDOFF = 4;
 
 // Per-row state written by the row kernels and read by the resolve kernel.
 struct RowStat {

@@ -167,14 +167,15 @@ __device__ void row_finished(const RowArgs &a, int r, unsigned char *scratch) {
                         skey + NUC_CAP, skey + 2 * NUC_CAP, skey + 3 * NUC_CAP, s_red, &s_draw);
 }
 
-// Hands row r to the general kernel with its max m (the row is finite: rows
-// with NaN or +inf were marked NONFINITE before any handoff), which spares
-// that kernel a pass.
-__device__ __forceinline__ void fallback_row(const RowArgs &a, int r, float m) {
+// Hands row r to the general kernel with its max m and its exp-sum S (in
+// units of 2^kref), which spare that kernel a pass and the exponentials of
+// another (the row is finite: rows with NaN or +inf were marked NONFINITE
+// before any handoff).
+__device__ __forceinline__ void fallback_row(const RowArgs &a, int r, float m, float kref, double S) {
     RowStat s;
     s.kref = m;
-    s.c = 0.f;
-    s.S_nuc = 0.0;
+    s.c = kref;
+    s.S_nuc = S;
     s.cut = 0ull;
     s.flags = RS_HANDOFF;
     s.nnuc = -1;
@@ -488,7 +489,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
         return;
     }
     if (bc < 0) {
-        if (tid == 0) fallback_row(a, r, m);
+        if (tid == 0) fallback_row(a, r, m, kref, S);
         return;
     }
     // ---- candidates: every id whose key reaches thr (bin <= bc) ----
@@ -543,7 +544,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     __syncthreads();
     const int ngl = s_ngl;
     if (ngl > CAND_CAP_F) {  // every listed group holds a candidate: too many
-        if (tid == 0) fallback_row(a, r, m);
+        if (tid == 0) fallback_row(a, r, m, kref, S);
         return;
     }
     // re-read the listed groups, one 16-byte chunk per thread and round;
@@ -575,7 +576,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     __syncthreads();
     const int n = s_ncand;
     if (n > CAND_CAP_F) {
-        if (tid == 0) fallback_row(a, r, m);
+        if (tid == 0) fallback_row(a, r, m, kref, S);
         return;
     }
     // ---- order the candidates (descending order value) into ord[] (the
@@ -653,7 +654,7 @@ __global__ void __launch_bounds__(NTF, 4) k_rows_fast(RowArgs a) {
     }
     __syncthreads();
     if (s_nstar == INT_MAX) {  // the candidates carry too little mass: exact path
-        if (tid == 0) fallback_row(a, r, m);
+        if (tid == 0) fallback_row(a, r, m, kref, S);
         return;
     }
     // keep the nucleus (in order) for the residual step when it fits

@@ -4,14 +4,18 @@
 // 16-byte aligned).  Masses are in 2^-40 fixed point, so every partial sum
 // is exact and order-independent.  One CTA of 512 threads per row; a
 // persistent grid walks the list of rows handed over by the fast kernel.
+//   value histogram  (aligned bfloat16 rows) ids counted per bfloat16 value
+//                below the max, the crossing and payload values found by a
+//                prefix scan, their ids collected and ranked: two row reads;
 //   binned path  exact per-bin masses over bins of distance below the max
 //                (warp-aggregated shared-memory atomics, farther elements
 //                summed in registers), then the crossing bin and the payload
-//                bins are collected and sorted: three to four row reads;
+//                bins are collected and ordered: three to four row reads;
 //   radix path   when a needed bin is too full or too far: exact radix
 //                selection over the 64-bit order value
 //                O = key(z) << 32 | (2^32 - 1 - id), 8 bits per pass.
 #include <climits>
+#include <type_traits>
 
 #include <cuda_bf16.h>
 
@@ -456,17 +460,18 @@ __device__ bool binned_row(const RowArgs &a, int r, const char *row, float m, fl
 // ---------------------------------------------------------------------------
 // Value-histogram path for bfloat16 rows.  A bfloat16 logit takes one of
 // 65536 values, and equal values have equal masses, so counting the elements
-// of each value is enough: the VH_W values below the row max get a count
-// (one shared-memory atomic per element, no per-element mass), and the
-// exp-sum S of the whole row is a compensated fp32 sum, as in the fast
-// kernel.  A prefix scan over the values then gives, exactly in 2^-40 fixed
-// point (count x the value's mass), the value holding the nucleus crossing
-// (first prefix reaching ceil(top_p * S * 2^40)) and the value holding the
-// k-th payload id; the elements of those values (ties are taken in id order,
-// which is the order-value order) are collected and ordered in shared
-// memory.  Returns false, having written nothing, when a needed value lies
-// below the window or a collected set exceeds VH_CAP; the binned path then
-// takes the row.
+// of each value is enough: the values of a window below the row max (at most
+// VH_W of them) get a count, one shared-memory atomic per element and no
+// per-element mass.  The exp-sum S of the whole row comes with a row handed
+// over by the fast kernel; otherwise the counting pass sums it in compensated
+// fp32, as the fast kernel does.  A prefix scan over the values then gives,
+// exactly in 2^-40 fixed point (count x the value's mass), the value holding
+// the nucleus crossing (first prefix reaching ceil(top_p * S * 2^40)) and the
+// value holding the k-th payload id; the elements of those values (ties are
+// taken in id order, which is the order-value order) are collected and ranked
+// in shared memory.  Returns false, having written nothing, when a needed
+// value lies below the window or a collected set exceeds VH_CAP; the binned
+// path then takes the row.
 constexpr int VH_W = 4096;    // values below the max with a count
 constexpr int VH_CAP = 1024;  // collected ids per set (payload values, crossing value)
 
@@ -480,14 +485,15 @@ struct ValHist {
     unsigned long long above_cut;      // the cut: order value of the crossing value's j-th id
 };
 
-// 16-bit order key of a bfloat16 value (the high half of fkey of the value,
-// with -0 taken as +0), and the value of a key
+// 16-bit order key of a bfloat16 value: 0x8000 plus the value's signed
+// magnitude, so keys sort like values and -0 and +0 share one key (-inf has
+// 0x80, the finite values 0x81..0xFF7F); and the value of a key
 __device__ __forceinline__ uint32_t bkey16(uint32_t b) {
-    b = b == 0x8000u ? 0u : b;
-    return (b & 0x8000u) ? (~b & 0xFFFFu) : (b | 0x8000u);
+    const uint32_t mag = b & 0x7FFFu;
+    return (b & 0x8000u) ? 0x8000u - mag : 0x8000u + mag;
 }
 __device__ __forceinline__ float bval16(uint32_t k) {
-    const uint32_t b = (k & 0x8000u) ? (k & 0x7FFFu) : (~k & 0xFFFFu);
+    const uint32_t b = k >= 0x8000u ? k - 0x8000u : (0x8000u | (0x8000u - k));
     return __uint_as_float(b << 16);
 }
 
@@ -506,15 +512,17 @@ __device__ __forceinline__ void warp_append_cap(unsigned long long *arr, int *n,
 }
 
 // (aligned bfloat16 rows; all threads of the CTA)
-// *n_fin_out gets the row's count of finite ids (computed by pass 1) even
-// when the row is declined.
-__device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, float kref,
+// S_in: the row's exp-sum in units of 2^kref for a row handed over by the
+// fast kernel, 0 otherwise.  *n_fin_out gets the row's count of finite ids
+// when top_p = 1 or S_in = 0 (its only uses), even when the row is declined.
+__device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, float kref, double S_in,
                             unsigned long long *n_fin_out, ValHist *vh, unsigned long long *buf, double *redd,
                             unsigned long long *redu) {
     using E = Elem<ACES_BF16>;
     const int tid = threadIdx.x, lane = tid & 31;
     const bool all_in = a.top_p >= 1.0f;
-    const uint32_t km = fkey(m) >> 16;  // m is a bfloat16 value: its 16-bit key
+    const bool have_S = S_in > 0.0;
+    const uint32_t km = bkey16(__float_as_uint(m) >> 16);  // m is a bfloat16 value
     for (int i = tid; i < VH_W; i += NT) vh->cnt[i] = 0u;
     if (tid == 0) {
         vh->npay = 0;
@@ -522,35 +530,63 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
         vh->dstar = all_in ? -1 : -2;  // -2: not (yet) found in the window
         vh->dk = -2;
     }
+    // the window: values km - d for d <= D (never -inf, whose key is 0x80)
+    uint32_t D = km - 0x81u < (uint32_t)(VH_W - 1) ? km - 0x81u : (uint32_t)(VH_W - 1);
+    if (have_S && !all_in) {
+        // Every id below a value of mass e_lo = (1 - top_p) S / (16 V) has
+        // less mass than that, so all of them together hold less than a
+        // sixteenth of the mass outside the nucleus and the crossing lies at
+        // or above that value; an id whose fixed-point mass is 0 (below
+        // 2^-40) is never needed either.  D is the last value reaching it.
+        const float g = fmaxf(log2f((1.0f - a.top_p) * (float)S_in / (16.0f * (float)a.V)), -41.0f);
+        const float vt = (kref + g) / a.c;
+        uint32_t lo = 0u, hi = D;  // bval16(km) = m >= vt
+        while (lo < hi) {
+            const uint32_t mid = (lo + hi + 1u) >> 1;
+            if (bval16(km - mid) >= vt) lo = mid;
+            else hi = mid - 1u;
+        }
+        D = lo;
+    }
     __syncthreads();
-    // ---- pass 1: counts per value and the compensated exp-sum ----
+    // ---- pass 1: counts per value (with the finite count and the
+    // compensated exp-sum where they are needed) ----
     float hi = 0.f, lo = 0.f;
     unsigned long long nfin = 0ull;
     const int nch = a.V / E::EPC;
-    for (int cc = tid; cc < nch; cc += NT) {
-        const uint4 w = ldg16(row + (size_t)cc * 16);
-        const uint32_t wd[4] = {w.x, w.y, w.z, w.w};
-        float cs = 0.f;
+    auto count_pass = [&](auto with_sum, auto with_nfin) {
+        constexpr bool WS = decltype(with_sum)::value, WN = decltype(with_nfin)::value;
+        for (int cc = tid; cc < nch; cc += NT) {
+            const uint4 w = ldg16(row + (size_t)cc * 16);
+            const uint32_t wd[4] = {w.x, w.y, w.z, w.w};
+            float cs = 0.f;
+            uint32_t nf = 0u;
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+            for (int q = 0; q < 4; ++q) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const uint32_t b = h ? (wd[q] >> 16) : (wd[q] & 0xFFFFu);
-                cs += ex2(fmaf(__uint_as_float(b << 16), a.c, -kref));  // 0 for -inf
-                const bool fin = b != 0xFF80u;
-                nfin += fin;
-                const uint32_t d = km - bkey16(b);
-                if (d < (uint32_t)VH_W && fin) atomicAdd(&vh->cnt[d], 1u);
+                for (int h = 0; h < 2; ++h) {
+                    const uint32_t b = h ? (wd[q] >> 16) : (wd[q] & 0xFFFFu);
+                    if (WS) cs += ex2(fmaf(__uint_as_float(b << 16), a.c, -kref));  // 0 for -inf
+                    if (WN) nf += b != 0xFF80u;
+                    const uint32_t d = km - bkey16(b);
+                    if (d <= D) atomicAdd(&vh->cnt[d], 1u);
+                }
+            }
+            if (WN) nfin += nf;
+            if (WS) {
+                const float t = hi + cs;  // Neumaier
+                if (fabsf(hi) >= fabsf(cs)) lo += (hi - t) + cs;
+                else lo += (cs - t) + hi;
+                hi = t;
             }
         }
-        const float t = hi + cs;  // Neumaier
-        if (fabsf(hi) >= fabsf(cs)) lo += (hi - t) + cs;
-        else lo += (cs - t) + hi;
-        hi = t;
-    }
-    const unsigned long long n_fin = block_reduce(nfin, redu, SumU64());
+    };
+    if (!have_S) count_pass(std::true_type(), std::true_type());
+    else if (all_in) count_pass(std::false_type(), std::true_type());
+    else count_pass(std::false_type(), std::false_type());
+    const unsigned long long n_fin = block_reduce(nfin, redu, SumU64());  // (its barriers order the counts)
     *n_fin_out = n_fin;
-    const double S = block_reduce((double)hi + (double)lo, redd, SumD());  // (its barriers order the counts)
+    const double S = have_S ? S_in : block_reduce((double)hi + (double)lo, redd, SumD());
     if (!(S > 0.0 && S < 1e300)) return false;
     const unsigned long long tg = all_in ? 0ull : (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
     // ---- prefix scan over the values, PER consecutive values per thread ----
@@ -612,23 +648,24 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
     if (dk >= 0 && vh->npay_need > (unsigned long long)VH_CAP) return false;
     if (dstar >= 0 && vh->cnt[dstar] > (uint32_t)VH_CAP) return false;
     // ---- collect every id of the values up to dk, and those of dstar ----
-    // (an id is taken only if its value reaches that of key km - max(dk,
-    // dstar): a chunk whose max is below it is skipped with one vote)
-    const float vthr = bval16(km - (uint32_t)(dk > dstar ? dk : dstar));
+    // A packed bfloat16 compare per pair of ids (value >= that of dk, or
+    // == that of dstar: IEEE order, where -0 == +0 as in the keys) lets a
+    // warp skip a round in which no id of its 32 chunks is wanted.
+    const float vk = dk >= 0 ? bval16(km - (uint32_t)dk) : INFINITY;
+    const float vs = dstar >= 0 ? bval16(km - (uint32_t)dstar) : NAN;
+    const __nv_bfloat162 vk2 = __floats2bfloat162_rn(vk, vk), vs2 = __floats2bfloat162_rn(vs, vs);
     for (int c0 = tid & ~31; c0 < nch; c0 += NT) {  // warp-uniform rounds
         const int c = c0 + lane;
         const bool in = c < nch;
         const uint4 w = in ? ldg16(row + (size_t)c * 16) : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
         const uint32_t wd[4] = {w.x, w.y, w.z, w.w};
-        {
-            const __nv_bfloat162 m2 = __hmax2(__hmax2(*reinterpret_cast<const __nv_bfloat162 *>(&wd[0]),
-                                                      *reinterpret_cast<const __nv_bfloat162 *>(&wd[1])),
-                                              __hmax2(*reinterpret_cast<const __nv_bfloat162 *>(&wd[2]),
-                                                      *reinterpret_cast<const __nv_bfloat162 *>(&wd[3])));
-            const uint32_t mu = *reinterpret_cast<const uint32_t *>(&m2);
-            const float cmax = fmaxf(__uint_as_float(mu << 16), __uint_as_float(mu & 0xFFFF0000u));
-            if (!__any_sync(0xffffffffu, in && cmax >= vthr)) continue;
+        uint32_t hm = 0u;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const __nv_bfloat162 x = *reinterpret_cast<const __nv_bfloat162 *>(&wd[q]);
+            hm |= __hge2_mask(x, vk2) | __heq2_mask(x, vs2);
         }
+        if (!__any_sync(0xffffffffu, hm != 0u)) continue;
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
 #pragma unroll
@@ -701,12 +738,16 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
     for (int idx = blockIdx.x; idx < nrows; idx += gridDim.x) {
         const int r = direct ? idx : a.ws.fb_list[idx];
         const char *row = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
-        // a row the fast kernel handed over comes with its max (and is finite)
-        const bool handed = DT == ACES_BF16 && VEC && !direct && a.ws.stats[r].flags == RS_HANDOFF;
+        // a row the fast kernel handed over comes with its max and its
+        // exp-sum (and is finite)
+        RowStat hs;
+        hs.flags = 0;
+        if (DT == ACES_BF16 && VEC && !direct) hs = a.ws.stats[r];
+        const bool handed = hs.flags == RS_HANDOFF;
         float m;
         unsigned long long n_fin = 0ull;
         if (handed) {
-            m = a.ws.stats[r].kref;
+            m = hs.kref;
         } else {
             // pass 0: max, finite count, invalid values
             if (tid == 0) s_bad = 0;
@@ -730,8 +771,11 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
         }
         const float kref = ceilf(m * a.c);  // masses are 2^(z*c - kref) <= 1
         if (DT == ACES_BF16 && VEC) {
+            // the handed exp-sum in units of 2^kref (its reference is the same
+            // ceil(m c); the power-of-two rescale is exact)
+            const double S_in = handed ? ldexp(hs.S_nuc, (int)(hs.c - kref)) : 0.0;
             unsigned long long nf = 0ull;
-            const bool done = valhist_row(a, r, row, m, kref, &nf, &paths.vh, buf, redd, redu);
+            const bool done = valhist_row(a, r, row, m, kref, S_in, &nf, &paths.vh, buf, redd, redu);
             __syncthreads();
             if (done) continue;
             n_fin = nf;
