@@ -474,6 +474,7 @@ __device__ bool binned_row(const RowArgs &a, int r, const char *row, float m, fl
 // path then takes the row.
 constexpr int VH_W = 4096;    // values below the max with a count
 constexpr int VH_CAP = 1024;  // collected ids per set (payload values, crossing value)
+constexpr int VH_U = 4;       // 16-byte loads per thread in flight in the counting pass
 
 struct ValHist {
     uint32_t cnt[VH_W];                // elements of value key16(max) - d
@@ -554,22 +555,31 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
     float hi = 0.f, lo = 0.f;
     unsigned long long nfin = 0ull;
     const int nch = a.V / E::EPC;
+    // (-inf words past the end count nowhere)
     auto count_pass = [&](auto with_sum, auto with_nfin) {
         constexpr bool WS = decltype(with_sum)::value, WN = decltype(with_nfin)::value;
-        for (int cc = tid; cc < nch; cc += NT) {
-            const uint4 w = ldg16(row + (size_t)cc * 16);
-            const uint32_t wd[4] = {w.x, w.y, w.z, w.w};
+        for (int c0 = tid; c0 < nch; c0 += VH_U * NT) {
+            uint4 wu[VH_U];
+#pragma unroll
+            for (int u = 0; u < VH_U; ++u) {
+                const int cc = c0 + u * NT;
+                wu[u] = cc < nch ? ldg16(row + (size_t)cc * 16) : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
+            }
             float cs = 0.f;
             uint32_t nf = 0u;
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
+            for (int u = 0; u < VH_U; ++u) {
+                const uint32_t wd[4] = {wu[u].x, wu[u].y, wu[u].z, wu[u].w};
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const uint32_t b = h ? (wd[q] >> 16) : (wd[q] & 0xFFFFu);
-                    if (WS) cs += ex2(fmaf(__uint_as_float(b << 16), a.c, -kref));  // 0 for -inf
-                    if (WN) nf += b != 0xFF80u;
-                    const uint32_t d = km - bkey16(b);
-                    if (d <= D) atomicAdd(&vh->cnt[d], 1u);
+                for (int q = 0; q < 4; ++q) {
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const uint32_t b = h ? (wd[q] >> 16) : (wd[q] & 0xFFFFu);
+                        if (WS) cs += ex2(fmaf(__uint_as_float(b << 16), a.c, -kref));  // 0 for -inf
+                        if (WN) nf += b != 0xFF80u;
+                        const uint32_t d = km - bkey16(b);
+                        if (d <= D) atomicAdd(&vh->cnt[d], 1u);
+                    }
                 }
             }
             if (WN) nfin += nf;
@@ -654,10 +664,13 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
     const float vk = dk >= 0 ? bval16(km - (uint32_t)dk) : INFINITY;
     const float vs = dstar >= 0 ? bval16(km - (uint32_t)dstar) : NAN;
     const __nv_bfloat162 vk2 = __floats2bfloat162_rn(vk, vk), vs2 = __floats2bfloat162_rn(vs, vs);
+    // (the next round's chunk is loaded before this round's ids are examined)
+    uint4 pw = tid < nch ? ldg16(row + (size_t)tid * 16) : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
     for (int c0 = tid & ~31; c0 < nch; c0 += NT) {  // warp-uniform rounds
         const int c = c0 + lane;
         const bool in = c < nch;
-        const uint4 w = in ? ldg16(row + (size_t)c * 16) : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
+        const uint4 w = pw;
+        pw = c + NT < nch ? ldg16(row + (size_t)(c + NT) * 16) : make_uint4(0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u, 0xFF80FF80u);
         const uint32_t wd[4] = {w.x, w.y, w.z, w.w};
         uint32_t hm = 0u;
 #pragma unroll
@@ -739,14 +752,15 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
         const int r = direct ? idx : a.ws.fb_list[idx];
         const char *row = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
         // a row the fast kernel handed over comes with its max and its
-        // exp-sum (and is finite)
+        // exp-sum (and is finite); the max pass runs only where the paths
+        // need the finite count it takes (top_p = 1 on float32 rows)
         RowStat hs;
         hs.flags = 0;
-        if (DT == ACES_BF16 && VEC && !direct) hs = a.ws.stats[r];
+        if (VEC && !direct) hs = a.ws.stats[r];
         const bool handed = hs.flags == RS_HANDOFF;
         float m;
         unsigned long long n_fin = 0ull;
-        if (handed) {
+        if (handed && (DT == ACES_BF16 || a.top_p < 1.0f)) {
             m = hs.kref;
         } else {
             // pass 0: max, finite count, invalid values
