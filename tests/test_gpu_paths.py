@@ -154,6 +154,27 @@ def test_value_histogram_ties(A, orc, n_vals, V, expect_valhist):
     assert res["checked_seqs"] >= 1
 
 
+def test_value_histogram_top_p_one_rows(A, orc):
+    # top_p = 1 on bf16 rows: 3000 ids spread over the sketch groups with
+    # values in [1, 1.05] (seven bf16 values, all within one sketch bin), the
+    # rest at -30.  The k-th id lies among ~3000 candidates, more than the
+    # fast kernel holds, so it hands every row over with its max and exp-sum;
+    # the value histogram counts the finite ids itself (the whole row is the
+    # nucleus) and takes the payload, ties in id order, from the top value.
+    V, n_hot = 64000, 3000
+    w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=1.0, k=64, seed=44)
+    rng = np.random.default_rng(44)
+    z = np.full((2, 2, V), -30.0, np.float32)
+    j = np.arange(n_hot)
+    ids = j * 16 + (j % 16)
+    for b in range(2):
+        for i in range(2):
+            z[b, i, ids] = rng.uniform(1.0, 1.05, n_hot).astype(np.float32)
+    counters, res = _run(A, orc, w, _bf16(z))
+    assert counters[0] == 4 and counters[6] == 4 and counters[4] == 0, counters
+    assert res["checked_seqs"] >= 1
+
+
 def test_signed_zeros_on_the_general_path(A, orc):
     # -0 and +0 are one value (one order key): the nucleus and the payload take
     # them in id order whatever their signs.  Ten positive ids, then a run of
