@@ -36,9 +36,14 @@ sys.path.insert(0, ROOT)
 METRIC = "verified rows/s and achieved HBM GB/s (fraction of GB300 peak) for verify+sparsify"
 WORKLOAD = "b256_k16_v256000_bf16"
 SWEEP_B = (32, 64, 128, 256)
-# kernels of one step: k_rows_fast, k_rows_general, k_resolve_seg,
-# k_resolve_pick (aces_verify), k_cache_build, k_cache_lookup
-KERNELS_PER_STEP = 6
+# kernels of one step: k_rows_cap, k_rows_general, k_resolve_cut,
+# k_resolve_seg, k_resolve_pick (aces_verify), k_cache_build, k_cache_lookup
+KERNELS_PER_STEP = 7
+VERIFY_KERNELS = ["k_rows_cap", "k_rows_general", "k_resolve_cut", "k_resolve_seg", "k_resolve_pick"]
+# path counters at the start of the workspace (int32 words)
+PATHS = ["rows_on_general_kernel", "timeouts", "rows_value_histogram", "rows_bitonic_order",
+         "general_rows_radix", "rows_cut_left_to_resolve", "general_rows_value_histogram",
+         "accept_tests_ranked_among_ties"]
 
 
 # ---------------------------------------------------------------------------
@@ -151,7 +156,7 @@ def measured_peak():
 
 # device code behind each profiled kernel (its file and the shared device header)
 KERNEL_SOURCES = {
-    "aces_verify": ("common.cuh", "rows_fast.cu", "rows_general.cu", "resolve.cu"),
+    "aces_verify": ("common.cuh", "rows_cap.cu", "rows_general.cu", "resolve.cu"),
     "k_cache_build": ("common.cuh", "cache.cu"),
 }
 
@@ -304,6 +309,100 @@ def cpu_baseline(w, inp):
                       f"({nseq * w.K} rows), OpenMP over sequences, {dt:.1f} s"}
 
 
+def oracle_rates(w, inp, seqs_all, seqs_one):
+    """The oracle as it stands on the machine's host cores: verify+sparsify rows/s
+    with every core (OpenMP over sequences) and with one thread, each on a
+    bounded sample of the workload's sequences."""
+    from oracle import oracle as O
+    O.build()
+    cores = O.num_threads()
+
+    def rate(nseq):
+        sub = {k: inp[k][:nseq] for k in ("z", "q", "xt", "u")}
+        t0 = time.perf_counter()
+        O.verify(sub["z"], sub["q"], sub["xt"], sub["u"], w.T, w.top_p, w.k)
+        dt = time.perf_counter() - t0
+        return nseq * (w.K + 1) / dt, dt
+
+    n_all = max(1, min(w.B, seqs_all, cores))
+    v_all, t_all = rate(n_all)
+    prev = O.set_threads(1)
+    try:
+        n_one = max(1, min(w.B, seqs_one))
+        v_one, t_one = rate(n_one)
+    finally:
+        O.set_threads(prev)
+    return {"value": v_all, "unit": "rows/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n_all} of {w.B} sequences ({n_all * (w.K + 1)} rows), verify+sparsify, {t_all:.2f} s",
+            "one_thread": {"value": v_one, "unit": "rows/s", "cores": 1,
+                           "sample": f"{n_one} sequence(s) ({n_one * (w.K + 1)} rows), {t_one:.2f} s"}}
+
+
+def per_config(A, torch, dev, stream, peak, peak_kind, have=None, cpu=True):
+    """aces_verify (k > 0) and aces_cache_build on every paper-shaped
+    workload at full size: CUDA-event times, algorithmic bytes, the fraction
+    of the measured HBM peak, the rows on each kernel path, and the oracle
+    timed beside it.  `have` maps a workload name to its already resident
+    inputs (host arrays, device tensors)."""
+    import gen
+    entries = []
+    for name, w in gen.WORKLOADS.items():
+        if have and name in have:
+            inp, d = have[name]
+        else:
+            inp = gen.generate_sequences(w, range(w.B), workers=min(16, os.cpu_count() or 1))
+            z = torch.from_numpy(inp["z"].view(np.int16)).view(torch.bfloat16) if w.dtype == "bf16" \
+                else torch.from_numpy(inp["z"])
+            d = {"z": z.to(dev), "q": torch.from_numpy(inp["q"]).to(dev),
+                 "xt": torch.from_numpy(inp["xt"]).to(dev), "u": torch.from_numpy(inp["u"]).to(dev)}
+        B, K, V, k = w.B, w.K, w.V, w.k
+        zsize = 2 if w.dtype == "bf16" else 4
+        wsb = torch.zeros(A.workspace_bytes(B, K, V, k), dtype=torch.uint8, device=dev)
+        out = A.verify(d["z"], d["q"], d["xt"], d["u"], w.T, w.top_p, k, workspace=wsb)
+        cache = A.cache_build(d["q"], d["xt"], w.F)
+        for _ in range(3):
+            A.verify(d["z"], d["q"], d["xt"], d["u"], w.T, w.top_p, k, out=out, workspace=wsb)
+        torch.cuda.synchronize()
+        n = 20
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+        for e0, e1 in ev:
+            e0.record(stream)
+            A.verify(d["z"], d["q"], d["xt"], d["u"], w.T, w.top_p, k, out=out, workspace=wsb)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        vms = statistics.median(e0.elapsed_time(e1) for e0, e1 in ev)
+        paths = dict(zip(PATHS, wsb[:32].view(torch.int32).cpu().numpy().tolist()))
+        paths.pop("timeouts")
+        vb = verify_bytes(B, K, V, k, zsize, resid_q_count(out, K, k))
+        for _ in range(3):
+            A.cache_build(d["q"], d["xt"], w.F, out=cache)
+        for e0, e1 in ev:
+            e0.record(stream)
+            A.cache_build(d["q"], d["xt"], w.F, out=cache)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        cms = statistics.median(e0.elapsed_time(e1) for e0, e1 in ev)
+        cb = cache_bytes(B, K, V, int(sum(w.F)))
+        rows = B * (K + 1)
+        gbs = vb / (vms * 1e-3) / 1e9
+        e = {"workload": name, "B": B, "K": K, "V": V, "logits": w.dtype, "T": w.T, "top_p": w.top_p, "k": k,
+             "F": list(w.F),
+             "verify_sparsify": {"ms": vms, "rows_per_s": rows / (vms * 1e-3), "alg_bytes": vb, "gbs": gbs,
+                                 "kernels": VERIFY_KERNELS, "paths": paths,
+                                 "l2": "logits %.1f MB %s the 129 MB L2; back-to-back calls" % (
+                                     rows * V * zsize / 1e6, "exceed" if rows * V * zsize > 129e6 else "fit in")},
+             "roofline_verify_sparsify": {"bound": "hbm", "kernel": "aces_verify", "achieved": gbs, "peak": peak,
+                                          "unit": "GB/s", "frac": gbs / peak, "peak_kind": peak_kind},
+             "cache_build": {"ms": cms, "alg_bytes": cb, "gbs": cb / (cms * 1e-3) / 1e9,
+                             "frac": cb / (cms * 1e-3) / 1e9 / peak, "kernels": ["k_cache_build"]}}
+        if cpu:
+            e["cpu_baseline"] = oracle_rates(w, inp, 16, 1)
+        entries.append(e)
+        del d, out, cache, wsb
+        torch.cuda.empty_cache()
+    return entries
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -318,6 +417,7 @@ def main():
                     help="skip the resample and KV-compaction timings (small profiling runs)")
     ap.add_argument("--e2e-steps", type=int, default=0)
     ap.add_argument("--B", type=int, default=0, help="use only the first B sequences (small profiling runs)")
+    ap.add_argument("--no-per-config", action="store_true", help="skip the five paper-shaped workloads' entries")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     ws, rank, local = init_dist()
@@ -424,16 +524,16 @@ def main():
     al = out["accept_len"].cpu().numpy()
     n_rej = int((al < K).sum())
     n_resid_q = resid_q_count(out, K, k)
-    fb = int(wsb[:4].view(torch.int32).item())
+    paths = dict(zip(PATHS, wsb[:32].view(torch.int32).cpu().numpy().tolist()))
+    paths.pop("timeouts")
     peak, peak_kind = measured_peak()
     vb = verify_bytes(B, K, V, k, zsize, n_resid_q)
     cb = cache_bytes(B, K, V, S)
     parts = {
         "verify_sparsify": {"ms": part_ms["verify_sparsify"], "rows_per_s": rows / (part_ms["verify_sparsify"] * 1e-3),
                             "alg_bytes": vb, "gbs": vb / (part_ms["verify_sparsify"] * 1e-3) / 1e9,
-                            "kernels": ["k_rows_fast", "k_rows_general", "k_resolve_seg",
-                                        "k_resolve_pick"],
-                            "rows_on_general_path": fb, "rejecting_sequences": n_rej},
+                            "kernels": VERIFY_KERNELS,
+                            "paths": paths, "rejecting_sequences": n_rej},
         "cache_build": {"ms": part_ms["cache_build"], "alg_bytes": cb,
                         "gbs": cb / (part_ms["cache_build"] * 1e-3) / 1e9, "kernels": ["k_cache_build"]},
         "cache_lookup": {"ms": part_ms["cache_lookup"], "kernels": ["k_cache_lookup"]},
@@ -491,6 +591,44 @@ def main():
                                "note": "KV [56, 64, 8, %d, 128] bf16; moved rows read + written; L2 flushed before each "
                                        "call; not part of the step" % S_kv}
         del kv
+    if not args.no_extras:
+        # the cache build at a fan-out of 64 per depth (one pass over q when
+        # the union of the per-thread lists proves the top 64), and on draft
+        # distributions of dense support (no min-p cut; the first 64 sequences)
+        def time_cache(qq, xx, FF, n=10):
+            o = A.cache_build(qq, xx, FF)
+            for _ in range(3):
+                A.cache_build(qq, xx, FF, out=o)
+            c0 = torch.cuda.Event(enable_timing=True)
+            c1 = torch.cuda.Event(enable_timing=True)
+            c0.record(stream)
+            for _ in range(n):
+                A.cache_build(qq, xx, FF, out=o)
+            c1.record(stream)
+            torch.cuda.synchronize()
+            return c0.elapsed_time(c1) / n
+        F64 = [64] * K
+        ms64 = time_cache(d["q"], d["xt"], F64)
+        cb64 = cache_bytes(B, K, V, 64 * K)
+        parts["cache_build_F64"] = {"ms": ms64, "alg_bytes": cb64, "gbs": cb64 / (ms64 * 1e-3) / 1e9,
+                                    "vs_F_of_the_step": ms64 / part_ms["cache_build"], "kernels": ["k_cache_build"],
+                                    "note": "F = [64] * K on the step's q; not part of the step"}
+        import dataclasses
+        bd = min(B, 64)
+        wd = dataclasses.replace(w, B=bd, draft_min_p=0.0)
+        dq = gen.generate_sequences(wd, shard(rank, bd), workers=min(16, os.cpu_count() or 1))
+        qd = torch.from_numpy(dq["q"]).to(dev)
+        xd = torch.from_numpy(dq["xt"]).to(dev)
+        msd = time_cache(qd, xd, list(w.F))
+        msd64 = time_cache(qd, xd, F64)
+        msm = time_cache(d["q"][:bd], d["xt"][:bd], list(w.F))
+        cbd = cache_bytes(bd, K, V, S)
+        parts["cache_build_dense_q"] = {
+            "sequences": bd, "ms": msd, "gbs": cbd / (msd * 1e-3) / 1e9, "ms_F64": msd64,
+            "ms_same_sequences_min_p_q": msm, "support": float((qd > 0).float().mean().item()),
+            "kernels": ["k_cache_build"],
+            "note": "q = tempered softmax of the draft logits with no support cut; not part of the step"}
+        del qd, xd, dq
     for p in parts.values():
         if "gbs" in p:
             p["frac_of_peak"] = p["gbs"] / peak
@@ -563,6 +701,13 @@ def main():
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w, inp)
 
+    # the five paper-shaped workloads, one entry each (N = 1 only)
+    pc = None
+    if rank == 0 and ws == 1 and not args.no_per_config:
+        del host, host_out, host_cache
+        have = {w.name: (inp, d)} if w.B == gen_B(w) else None
+        pc = per_config(A, torch, dev, stream, peak, peak_kind, have=have, cpu=not args.no_cpu_baseline)
+
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "rows/s", "n_gpus": ws, "steps": args.steps,
@@ -570,6 +715,7 @@ def main():
             "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": config_of(w),
             "roofline": roof, "roofline_verify_sparsify": roof_v, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": KERNELS_PER_STEP * args.steps, "clocks": clocks.summary(), "parts": parts, "sweep": sweep,
+            "per_config": pc,
         }
         print(json.dumps(line), flush=True)
     if pg is not None:

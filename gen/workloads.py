@@ -14,9 +14,10 @@ Recipe (per sequence, positions i = 0..K):
   * logits are rounded to float32 (and then to bfloat16, round-to-nearest-
     even, for bf16 workloads)
   * draft distribution q[i, :] for i < K: tempered weights
-    exp((zd - max zd) / T) restricted to ids whose weight is >= 1e-4 of the
-    largest (a min-p style support cut of the draft sampler), normalised,
-    stored as float32.  This stands in for the edge model's output Q.
+    exp((zd - max zd) / T) restricted to ids whose weight is >= draft_min_p
+    (1e-4 by default) of the largest (a min-p style support cut of the draft
+    sampler; 0 keeps every id), normalised, stored as float32.  This stands
+    in for the edge model's output Q.
   * draft token x~[i] is drawn from the float32 q[i] by inverse CDF.
   * uniforms u[i] for i <= K are float32 in (0, 1): u[:, i<K] drive the
     accept tests and u[:, K] the single residual / bonus draw.
@@ -51,6 +52,7 @@ class Workload:
     k: int
     F: tuple
     seed: int
+    draft_min_p: float = 1e-4  # support cut of the draft sampler (0: every id keeps q > 0)
 
     @property
     def rows(self) -> int:
@@ -100,8 +102,9 @@ def _zipf_head(w: Workload):
     return ids, bias
 
 
-def _one_sequence(w: Workload, b: int, head):
-    """Returns (z float32 [K+1,V], q float32 [K,V], xt int32 [K], u float32 [K+1])."""
+def _one_sequence(w: Workload, b: int, head, draft_logits: bool = False):
+    """Returns (z float32 [K+1,V], q float32 [K,V], xt int32 [K], u float32 [K+1]),
+    plus the draft logits zd float32 [K+1,V] when draft_logits is set."""
     rng = np.random.Generator(np.random.Philox(np.random.SeedSequence([w.seed, b])))
     K, V = w.K, w.V
     big = V >= 100000
@@ -123,7 +126,8 @@ def _one_sequence(w: Workload, b: int, head):
     for i in range(K):
         d = zd[i].astype(np.float64)
         wgt = np.exp((d - d.max()) / w.T)
-        wgt[wgt < DRAFT_MIN_P] = 0.0
+        if w.draft_min_p > 0.0:
+            wgt[wgt < w.draft_min_p] = 0.0
         q[i] = (wgt / wgt.sum()).astype(np.float32)
         c = np.cumsum(q[i], dtype=np.float64)
         t = rng.random() * c[-1]
@@ -133,6 +137,8 @@ def _one_sequence(w: Workload, b: int, head):
             j -= 1
         xt[i] = j
     u = (rng.integers(1, 1 << 24, size=K + 1).astype(np.float64) / float(1 << 24)).astype(np.float32)
+    if draft_logits:
+        return z32, q, xt, u, zd.astype(np.float32)
     return z32, q, xt, u
 
 
@@ -172,12 +178,15 @@ def _fill(args):
     return len(seqs)
 
 
-def generate_sequences(name, seqs: Sequence[int], workers: int = 0, B: Optional[int] = None):
+def generate_sequences(name, seqs: Sequence[int], workers: int = 0, B: Optional[int] = None,
+                       draft_logits: bool = False):
     """Generate the listed sequences of workload `name` (a name or a Workload).
 
     Returns a dict with z ([n,K+1,V] float32, or uint16 bfloat16 bits), q
-    ([n,K,V] float32), xt ([n,K] int32), u ([n,K+1] float32) and the workload.
-    `workers` > 1 uses a spawn-started process pool (safe after CUDA init).
+    ([n,K,V] float32), xt ([n,K] int32), u ([n,K+1] float32) and the workload;
+    with draft_logits also zd ([n,K+1,V] float32, the draft logits q was
+    made from; one process).  `workers` > 1 uses a spawn-started process
+    pool (safe after CUDA init).
     """
     w = _resolve(name)
     seqs = [int(s) for s in seqs]
@@ -185,15 +194,22 @@ def generate_sequences(name, seqs: Sequence[int], workers: int = 0, B: Optional[
     zdt = np.uint16 if w.dtype == "bf16" else np.float32
     shapes = [((n, w.K + 1, w.V), zdt), ((n, w.K, w.V), np.float32),
               ((n, w.K), np.int32), ((n, w.K + 1), np.float32)]
-    if workers <= 1 or n < 4:
+    if workers <= 1 or n < 4 or draft_logits:
         head = _zipf_head(w) if w.zipf else None
         z = np.empty(*shapes[0]); q = np.empty(*shapes[1])
         xt = np.empty(*shapes[2]); u = np.empty(*shapes[3])
+        zd = np.empty((n, w.K + 1, w.V), np.float32) if draft_logits else None
         for pos, b in enumerate(seqs):
-            zz, qq, xx, uu = _one_sequence(w, b, head)
+            r = _one_sequence(w, b, head, draft_logits)
+            zz, qq, xx, uu = r[:4]
             z[pos] = f32_to_bf16(zz) if w.dtype == "bf16" else zz
             q[pos] = qq; xt[pos] = xx; u[pos] = uu
-        return dict(z=z, q=q, xt=xt, u=u, w=w, seqs=np.array(seqs))
+            if draft_logits:
+                zd[pos] = r[4]
+        out = dict(z=z, q=q, xt=xt, u=u, w=w, seqs=np.array(seqs))
+        if draft_logits:
+            out["zd"] = zd
+        return out
     import multiprocessing as mp
     from multiprocessing import shared_memory
     shms = [shared_memory.SharedMemory(create=True, size=max(1, int(np.prod(s)) * np.dtype(d).itemsize))

@@ -83,12 +83,12 @@ typedef struct CUstream_st *aces_stream_t;
 
 /*
  * Bytes of device scratch that aces_verify (B sequences, K >= 1) or
- * aces_sparsify (B rows, K = 0) needs: about 4.1 KiB per target row for
- * aces_verify, under 100 bytes per row for aces_sparsify, plus, for both,
- * room to split up to 640 rows over several CTAs (about V / 4 + 8.3 KiB per
- * row; 64 MB in all at B = 256, K = 16, V = 256000).  The caller allocates
- * it, passes it to the call and must not use it while the call's work is in
- * flight; it needs no initialisation.  Returns 0 for invalid sizes.
+ * aces_sparsify (B rows, K = 0) needs: about 4.2 KiB per target row for
+ * aces_verify (almost all of it the row's nucleus, kept for the residual
+ * draw when it has at most 512 ids), under 100 bytes per row for
+ * aces_sparsify.  The caller allocates it, passes it to the call and must
+ * not use it while the call's work is in flight; it needs no
+ * initialisation.  Returns 0 for invalid sizes.
  */
 size_t aces_workspace_bytes(int B, int K, int V, int k);
 
@@ -119,8 +119,7 @@ size_t aces_workspace_bytes(int B, int K, int V, int k);
  * workspace / workspace_bytes: device scratch of at least
  *   aces_workspace_bytes(B, K, V, k) bytes, 16-byte aligned.  It includes
  *   4 KiB per row to keep each row's nucleus (when it has at most 512 ids)
- *   for the residual draw, which then reads q at those ids only, and the
- *   areas through which the CTAs sharing a split row combine their parts.
+ *   for the residual draw, which then reads q at those ids only.
  * Limits: 1 <= B, 1 <= K <= ACES_MAX_K, 2 <= V <= ACES_MAX_V,
  *   0 <= k <= min(V, ACES_MAX_TOPK).
  */
@@ -145,12 +144,11 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
  * library, kept on every GPU that loads the library until the process exits.
  * This call allocates nothing.
  *   - Size limit: returns ACES_ERR_UNSUPPORTED (nothing launched) when
- *     B > 981 at K = 16, B > 1401 at K = 8, B > 1783 at K = 4 (the limit
+ *     B > 923 at K = 16, B > 1284 at K = 8, B > 1598 at K = 4 (the limit
  *     does not depend on V or k).  The scratch keeps nucleus lists only for
  *     B <= 14 at K = 16 (27 at K = 8, 49 at K = 4); without them the
- *     residual draw scans its whole row.  It splits rows over CTAs only when
- *     aces_workspace_bytes(B, K, V, k) fits in it (B <= 3 at K = 16 for
- *     V = 32000).  The results are the same either way.
+ *     residual draw scans its whole row.  The results are the same either
+ *     way.
  *   - Set-up: the first call on each device looks up the array's device
  *     address (cudaGetSymbolAddress) with that device current; make that
  *     first call before any stream capture on the device.
@@ -158,6 +156,8 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
  *     last call's contents (each call clears what it needs).  Calls whose
  *     work overlaps on the GPU race on it: serialize them (one stream, or
  *     events between streams).
+ *   - The looked-up address is kept for the life of the process: no
+ *     cudaDeviceReset may come between two calls on a device.
  */
 #define ACES_NOALLOC_SCRATCH_BYTES (1 << 20)
 aces_status aces_verify_noalloc(const void *target_logits, aces_dtype dt, const float *draft_probs,
@@ -165,6 +165,20 @@ aces_status aces_verify_noalloc(const void *target_logits, aces_dtype dt, const 
                                 int V, float T, float top_p, int32_t *accept_len,
                                 int32_t *out_token, int k, int32_t *topk_ids, float *topk_probs,
                                 float *tail_mass, int32_t *row_status, aces_stream_t stream);
+
+/*
+ * aces_verify on the library's exact general row kernel alone: the same
+ * arguments, outputs, limits, errors and results (bit for bit), but every
+ * row takes the slow path that aces_verify keeps for rows its single-pass
+ * kernel cannot settle (it reads each row two to four times).  A reference
+ * for checking the fast path; not meant for serving.
+ */
+aces_status aces_verify_exact(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                              const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                              float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                              int32_t *topk_ids, float *topk_probs, float *tail_mass,
+                              int32_t *row_status, void *workspace, size_t workspace_bytes,
+                              aces_stream_t stream);
 
 /*
  * Sparse payload alone for `rows` independent target rows (the COMPRESS of
@@ -332,6 +346,19 @@ aces_status aces_tree_budget(const double *draft_latency_s, int n, double rtt_s,
  * 1 <= gamma <= ACES_MAX_K.  Host-only; launches nothing.
  */
 aces_status aces_branch_alloc(int B_alloc, int gamma, double alpha, double beta, int32_t *F_out);
+
+#ifdef ACES_CHECKED
+/*
+ * Checked build only (compiled with -DACES_CHECKED; a test aid, not part of
+ * the product library): every kernel checks its data-dependent shared- and
+ * global-memory indices and records the first index out of range instead of
+ * making the access.  This returns that record since the last call:
+ * out[0] = site (source file number * 10000 + line; 0 when none), out[1] =
+ * the index, out[2] = its bound.  It waits for the device and clears the
+ * record.  The paper has no counterpart.
+ */
+aces_status aces_checked_violation(unsigned long long out[3]);
+#endif
 
 /* Static English text for a status code. */
 const char *aces_status_string(aces_status s);

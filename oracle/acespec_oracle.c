@@ -646,3 +646,17 @@ int orc_num_threads(void) {
     return 1;
 #endif
 }
+
+/* Threads of the parallel loops that follow (n >= 1); returns the previous
+ * count.  The results do not depend on it (every loop is over independent
+ * rows or sequences). */
+int orc_set_threads(int n) {
+#ifdef _OPENMP
+    const int prev = omp_get_max_threads();
+    if (n >= 1) omp_set_num_threads(n);
+    return prev;
+#else
+    (void)n;
+    return 1;
+#endif
+}

@@ -62,8 +62,9 @@ def _load():
             lib.orc_hit_prob.argtypes = [P, P, P, I, I, I, D, D, P, P, P, P]
             lib.orc_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P, P, P, P, P]
             lib.orc_num_threads.argtypes = []
+            lib.orc_set_threads.argtypes = [I]
             for f in (lib.orc_sparsify, lib.orc_verify, lib.orc_cache_build, lib.orc_cache_lookup,
-                      lib.orc_num_threads):
+                      lib.orc_num_threads, lib.orc_set_threads):
                 f.restype = I
             _lib = lib
     return _lib
@@ -81,6 +82,11 @@ def _logits_f32(z: np.ndarray) -> np.ndarray:
 
 def num_threads() -> int:
     return int(_load().orc_num_threads())
+
+
+def set_threads(n: int) -> int:
+    """Threads of the oracle's parallel loops from now on; returns the previous count."""
+    return int(_load().orc_set_threads(int(n)))
 
 
 def sparsify(z, T: float, top_p: float, k: int):

@@ -21,13 +21,15 @@ import threading
 
 import torch
 
-__all__ = ["load", "lib_path", "workspace_bytes", "verify", "sparsify", "cache_build", "cache_lookup",
+__all__ = ["load", "use_checked", "checked_violation", "lib_path", "workspace_bytes", "verify", "sparsify", "cache_build", "cache_lookup",
            "ROW_NONFINITE", "ROW_BAD_Q", "AcespecError"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "libacespec.so")
+_LIB_CHECKED = os.path.join(_HERE, "libacespec_checked.so")
 _lock = threading.Lock()
-_lib = None
+_lib = None          # the library every function below calls
+_libs = {}           # loaded libraries by path
 
 ROW_NONFINITE = 1
 ROW_BAD_Q = 2
@@ -50,34 +52,65 @@ def load():
     """Load libacespec.so (built by __graft_entry__.build() or build.py)."""
     global _lib
     with _lock:
-        if _lib is not None:
-            return _lib
-        if not os.path.exists(_LIB_PATH):
-            raise RuntimeError(f"{_LIB_PATH} is missing: build it with `python -m paper_2609_02514_gb300.build`")
-        lib = ctypes.CDLL(_LIB_PATH)
-        P, I, F, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
-        lib.aces_workspace_bytes.argtypes = [I, I, I, I]
-        lib.aces_workspace_bytes.restype = S
-        lib.aces_verify.argtypes = [P, I, P, P, P, I, I, I, F, F, P, P, I, P, P, P, P, P, S, P]
-        lib.aces_sparsify.argtypes = [P, I, I, I, F, F, I, P, P, P, P, P, S, P]
-        lib.aces_cache_build.argtypes = [P, P, P, I, I, I, P, P, P]
-        lib.aces_cloud_step.argtypes = [P, I, P, P, P, I, I, I, F, F, P, P, I, P, P, P, P, P, P, P, P, S, P]
-        lib.aces_cache_lookup.argtypes = [P, P, I, I, P, P, P, P]
-        lib.aces_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P]
-        lib.aces_compact_kv.argtypes = [P, I, I, I, I, I, I, P, P, P, I, I, P, P]
-        lib.aces_tree_tokens.argtypes = [P, I, I]
-        lib.aces_tree_tokens.restype = I
-        lib.aces_tree_mask.argtypes = [P, I, I, P, P, P]
-        lib.aces_tree_budget.argtypes = [P, I, ctypes.c_double, ctypes.c_double, I, P]
-        lib.aces_branch_alloc.argtypes = [I, I, ctypes.c_double, ctypes.c_double, P]
-        lib.aces_status_string.argtypes = [I]
-        lib.aces_status_string.restype = ctypes.c_char_p
-        for f in (lib.aces_verify, lib.aces_sparsify, lib.aces_cache_build, lib.aces_cache_lookup,
-                  lib.aces_resample_sparse, lib.aces_tree_budget, lib.aces_branch_alloc,
-                  lib.aces_compact_kv, lib.aces_tree_mask):
-            f.restype = I
-        _lib = lib
-        return lib
+        if _lib is None:
+            _lib = _open(_LIB_PATH)
+        return _lib
+
+
+def use_checked(on: bool = True):
+    """Route every call of this module to the checked test build,
+    libacespec_checked.so (built with build.build(checked=True)), or back to
+    the product library.  Returns the library now in use."""
+    global _lib
+    with _lock:
+        _lib = _open(_LIB_CHECKED if on else _LIB_PATH)
+        return _lib
+
+
+def checked_violation():
+    """(site, index, bound) of the first out-of-range index the checked
+    build met since the last call, or None; clears the record."""
+    lib = load()
+    if not hasattr(lib, "aces_checked_violation"):
+        raise RuntimeError("the product library has no index checks: call use_checked() first")
+    out = (ctypes.c_ulonglong * 3)()
+    _check("aces_checked_violation", lib.aces_checked_violation(out))
+    return None if out[0] == 0 else (int(out[0]), int(out[1]), int(out[2]))
+
+
+def _open(path):
+    if path in _libs:
+        return _libs[path]
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with `python -m paper_2609_02514_gb300.build`")
+    lib = ctypes.CDLL(path)
+    P, I, F, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+    lib.aces_workspace_bytes.argtypes = [I, I, I, I]
+    lib.aces_workspace_bytes.restype = S
+    lib.aces_verify.argtypes = [P, I, P, P, P, I, I, I, F, F, P, P, I, P, P, P, P, P, S, P]
+    lib.aces_verify_exact.argtypes = lib.aces_verify.argtypes
+    lib.aces_sparsify.argtypes = [P, I, I, I, F, F, I, P, P, P, P, P, S, P]
+    lib.aces_cache_build.argtypes = [P, P, P, I, I, I, P, P, P]
+    lib.aces_cloud_step.argtypes = [P, I, P, P, P, I, I, I, F, F, P, P, I, P, P, P, P, P, P, P, P, S, P]
+    lib.aces_cache_lookup.argtypes = [P, P, I, I, P, P, P, P]
+    lib.aces_resample_sparse.argtypes = [P, P, P, P, P, P, P, I, I, I, I, P, P, P]
+    lib.aces_compact_kv.argtypes = [P, I, I, I, I, I, I, P, P, P, I, I, P, P]
+    lib.aces_tree_tokens.argtypes = [P, I, I]
+    lib.aces_tree_tokens.restype = I
+    lib.aces_tree_mask.argtypes = [P, I, I, P, P, P]
+    lib.aces_tree_budget.argtypes = [P, I, ctypes.c_double, ctypes.c_double, I, P]
+    lib.aces_branch_alloc.argtypes = [I, I, ctypes.c_double, ctypes.c_double, P]
+    lib.aces_status_string.argtypes = [I]
+    lib.aces_status_string.restype = ctypes.c_char_p
+    for f in (lib.aces_verify, lib.aces_verify_exact, lib.aces_sparsify, lib.aces_cache_build,
+              lib.aces_cache_lookup, lib.aces_resample_sparse, lib.aces_tree_budget, lib.aces_branch_alloc,
+              lib.aces_compact_kv, lib.aces_tree_mask):
+        f.restype = I
+    if hasattr(lib, "aces_checked_violation"):
+        lib.aces_checked_violation.argtypes = [P]
+        lib.aces_checked_violation.restype = I
+    _libs[path] = lib
+    return lib
 
 
 def _check(fn, code):
@@ -114,7 +147,7 @@ def workspace_bytes(B: int, K: int, V: int, k: int) -> int:
 
 
 def verify(target_logits, draft_probs, draft_tokens, uniforms, T: float, top_p: float, k: int = 0,
-           out: dict | None = None, workspace: torch.Tensor | None = None):
+           out: dict | None = None, workspace: torch.Tensor | None = None, exact: bool = False):
     """Lossless verification of B drafted chains (+ sparse payload when k > 0).
 
     target_logits [B, K+1, V] float32/bfloat16, draft_probs [B, K, V] float32,
@@ -122,6 +155,8 @@ def verify(target_logits, draft_probs, draft_tokens, uniforms, T: float, top_p: 
     Returns a dict of device tensors: accept_len [B], out_token [B],
     row_status [B, K+1] and, when k > 0, topk_ids / topk_probs [B, K+1, k],
     tail_mass [B, K+1].  `out` may supply preallocated outputs (same keys).
+    exact=True calls aces_verify_exact (every row on the exact general
+    kernel; same results, slower).
     """
     lib = load()
     z = _cuda(target_logits, "target_logits")
@@ -151,11 +186,12 @@ def verify(target_logits, draft_probs, draft_tokens, uniforms, T: float, top_p: 
         o.setdefault("tail_mass", torch.empty(B, R, **f32))
     need = workspace_bytes(B, K, V, k)
     ws = workspace if workspace is not None else torch.empty(max(need, 16), dtype=torch.uint8, device=dev)
-    code = lib.aces_verify(_p(z), _dtype_code(z), _p(q), _p(xt), _p(u), B, K, V, float(T), float(top_p),
-                           _p(o["accept_len"]), _p(o["out_token"]), int(k), _p(o.get("topk_ids")),
-                           _p(o.get("topk_probs")), _p(o.get("tail_mass")), _p(o["row_status"]),
-                           _p(ws), ws.numel(), _stream(dev))
-    _check("aces_verify", code)
+    fn = lib.aces_verify_exact if exact else lib.aces_verify
+    code = fn(_p(z), _dtype_code(z), _p(q), _p(xt), _p(u), B, K, V, float(T), float(top_p),
+              _p(o["accept_len"]), _p(o["out_token"]), int(k), _p(o.get("topk_ids")),
+              _p(o.get("topk_probs")), _p(o.get("tail_mass")), _p(o["row_status"]),
+              _p(ws), ws.numel(), _stream(dev))
+    _check("aces_verify_exact" if exact else "aces_verify", code)
     return o
 
 

@@ -2,7 +2,9 @@
 
 Each translation unit is compiled in parallel with nvcc, then linked into one
 shared library (CUDA runtime linked statically).  Re-running is a no-op when
-the library is newer than every source.
+the library is newer than every source.  build(checked=True) makes the
+checked test build instead, libacespec_checked.so (-DACES_CHECKED: every
+kernel records out-of-range indices instead of using them).
 """
 from __future__ import annotations
 
@@ -16,6 +18,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 LIB = os.path.join(HERE, "libacespec.so")
+LIB_CHECKED = os.path.join(HERE, "libacespec_checked.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2"]
 
@@ -36,25 +39,26 @@ def _deps():
         os.path.join(ROOT, "include", "acespec.h")]
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def up_to_date(lib: str = LIB) -> bool:
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(p) <= t for p in _deps())
 
 
-def build(force: bool = False, verbose: bool = False) -> str:
-    if not force and up_to_date():
-        return LIB
+def build(force: bool = False, verbose: bool = False, checked: bool = False) -> str:
+    lib = LIB_CHECKED if checked else LIB
+    if not force and up_to_date(lib):
+        return lib
     nvcc = _nvcc()
-    bdir = os.path.join(HERE, "_build")
+    bdir = os.path.join(HERE, "_build_checked" if checked else "_build")
     os.makedirs(bdir, exist_ok=True)
     procs = []
     objs = []
     for src in _sources():
         obj = os.path.join(bdir, os.path.basename(src)[:-3] + ".o")
         objs.append(obj)
-        cmd = [nvcc] + ARCH + FLAGS + ["-c", src, "-o", obj]
+        cmd = [nvcc] + ARCH + FLAGS + (["-DACES_CHECKED"] if checked else []) + ["-c", src, "-o", obj]
         procs.append((cmd, subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT)))
     for cmd, p in procs:
         out, _ = p.communicate()
@@ -62,14 +66,14 @@ def build(force: bool = False, verbose: bool = False) -> str:
             raise RuntimeError("nvcc failed: " + " ".join(cmd) + "\n" + out.decode(errors="replace"))
         if verbose and out:
             sys.stdout.write(out.decode(errors="replace"))
-    tmp = LIB + f".tmp{os.getpid()}"
+    tmp = lib + f".tmp{os.getpid()}"
     link = [nvcc] + ARCH + ["-shared", "-o", tmp] + objs
     r = subprocess.run(link, capture_output=True)
     if r.returncode != 0:
         raise RuntimeError("link failed: " + " ".join(link) + "\n" + r.stdout.decode() + r.stderr.decode())
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose=True))
+    print(build(force="--force" in sys.argv, verbose=True, checked="--checked" in sys.argv))

@@ -4,6 +4,7 @@
 #include <cmath>
 #include <mutex>
 
+#define ACES_FILE 1  // site numbers of the checked build
 #include "common.cuh"
 
 using namespace aces;
@@ -39,45 +40,24 @@ aces_status check_rows(const void *logits, aces_dtype dt, long long rows, int V,
     return ACES_OK;
 }
 
-// Row kernels: fast sketch path when rows are 16-byte aligned, then the
-// exact general path for every row the fast path handed over.
-aces_status run_rows(RowArgs &a, aces_dtype dt, cudaStream_t s) {
+// Row kernels: the single-pass capture kernel when rows are 16-byte
+// aligned, then the exact general kernel for every row it handed over (or
+// for every row otherwise).
+aces_status run_rows(RowArgs &a, aces_dtype dt, bool exact, cudaStream_t s) {
     const size_t es = elem_size(dt);
     const bool vec = aligned16(a.logits) && ((size_t)a.V * es) % 16 == 0;
     const int nsm = sm_count();
     const int nseq = a.K > 0 ? a.rows / (a.K + 1) : a.rows;
-    if (cudaMemsetAsync(a.ws.fb_count, 0, ws_clear_bytes(nseq, a.K, a.ws.parts != nullptr), s) != cudaSuccess)
-        return ACES_ERR_CUDA;
-    const int gc = vec ? rows_fast_gc(dt, a.V) : 0;
-    if (gc > 0) {
-        const int nch = (int)((size_t)a.V * es / 16);
-        a.ng = (nch + gc - 1) / gc;  // sketch groups of gc 16-byte chunks
-        const size_t smem = rows_fast_smem(dt, gc, nch);
-        // Split the rows of the last partial wave (every row of a batch
-        // smaller than one wave) over 2 or 4 CTAs, so the SMs stay busy at
-        // the end of the launch.
-        a.r_full = a.rows;
-        a.P = 1;
-        a.gper = a.ng;
-        const long long slots = (long long)rows_fast_per_sm(dt, gc, smem) * nsm;
-        if (a.ws.parts != nullptr && slots > 0) {
-            const long long rr = a.rows < slots ? a.rows : a.rows % slots;
-            if (rr > 0 && rr <= SPLIT_ROWS_MAX) {
-                a.P = 4 * rr <= slots ? 4 : 2;
-                a.r_full = a.rows - (int)rr;
-                a.gper = (a.ng + a.P - 1) / a.P;
-            }
-        }
-        if (launch_rows_fast(a, dt, gc, smem, s) != cudaSuccess) return ACES_ERR_CUDA;
-        int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
+    if (cudaMemsetAsync(a.ws.fb_count, 0, ws_clear_bytes(nseq, a.K), s) != cudaSuccess) return ACES_ERR_CUDA;
+    const int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
+    if (vec) {
+        rows_cap_layout(a, dt);
+        a.force_fb = exact ? 1 : 0;
+        if (launch_rows_cap(a, dt, s) != cudaSuccess) return ACES_ERR_CUDA;
         if (launch_rows_general(a, dt, true, 0, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
     } else {
-        a.ng = 0;
-        a.r_full = a.rows;
-        a.P = 1;
-        a.gper = 0;
-        int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
-        if (launch_rows_general(a, dt, vec, 1, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
+        a.force_fb = 0;
+        if (launch_rows_general(a, dt, false, 1, grid, s) != cudaSuccess) return ACES_ERR_CUDA;
     }
     return ACES_OK;
 }
@@ -91,7 +71,7 @@ size_t aces_workspace_bytes(int B, int K, int V, int k) {
         return 0;
     long long rows = (long long)B * (K + 1);
     if (rows > INT_MAX / 2) return 0;
-    return ws_bytes((int)rows, B, K, true, true, V);
+    return ws_bytes((int)rows, B, K, true);
 }
 
 }  // extern "C"
@@ -101,29 +81,30 @@ static aces_status verify_check(const void *target_logits, aces_dtype dt, const 
                                 const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
                                 float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
                                 int32_t *topk_ids, float *topk_probs, float *tail_mass, int32_t *row_status,
-                                void *workspace, size_t workspace_bytes, bool lists, bool split) {
+                                void *workspace, size_t workspace_bytes, bool lists) {
     if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
     aces_status st = check_rows(target_logits, dt, (long long)B * (K + 1), V, T, top_p, k, false,
                                 topk_ids, topk_probs, tail_mass, row_status);
     if (st != ACES_OK) return st;
     if (!draft_probs || !draft_tokens || !uniforms || !accept_len || !out_token || !workspace)
         return ACES_ERR_INVALID_ARG;
-    if (!aligned16(workspace) || workspace_bytes < ws_bytes(B * (K + 1), B, K, lists, split, V))
+    if (!aligned16(workspace) || workspace_bytes < ws_bytes(B * (K + 1), B, K, lists))
         return ACES_ERR_INVALID_ARG;
     return ACES_OK;
 }
 
 // Results depend on neither `lists` (without them the residual draw scans its
-// whole row instead of the stored nucleus) nor `split`.
+// whole row instead of the stored nucleus) nor `exact` (every row on the
+// general kernel).
 aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const float *draft_probs,
                         const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
                         float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
                         int32_t *topk_ids, float *topk_probs, float *tail_mass,
                         int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
-                        bool split, aces_stream_t stream) {
+                        bool exact, aces_stream_t stream) {
     aces_status st = verify_check(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
                                   accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status,
-                                  workspace, workspace_bytes, lists, split);
+                                  workspace, workspace_bytes, lists);
     if (st != ACES_OK) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     const int rows = B * (K + 1);
@@ -144,11 +125,10 @@ aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const fl
     a.topk_probs = topk_probs;
     a.tail = tail_mass;
     a.row_status = row_status;
-    a.ws = ws_carve(workspace, rows, B, K, lists && top_p < 1.0f, split, V);
+    a.ws = ws_carve(workspace, rows, B, K, lists && top_p < 1.0f);
     a.accept_len = accept_len;
     a.out_token = out_token;
-    a.ng = 0;
-    st = run_rows(a, dt, s);
+    st = run_rows(a, dt, exact, s);
     if (st != ACES_OK) return st;
     ResolveArgs r;
     r.logits = target_logits;
@@ -175,6 +155,19 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
                         int32_t *topk_ids, float *topk_probs, float *tail_mass,
                         int32_t *row_status, void *workspace, size_t workspace_bytes,
                         aces_stream_t stream) {
+    if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
+    if (workspace_bytes < aces_workspace_bytes(B, K, V, k)) return ACES_ERR_INVALID_ARG;
+    return verify_impl(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
+                       accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status,
+                       workspace, workspace_bytes, true, false, stream);
+}
+
+aces_status aces_verify_exact(const void *target_logits, aces_dtype dt, const float *draft_probs,
+                              const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
+                              float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
+                              int32_t *topk_ids, float *topk_probs, float *tail_mass,
+                              int32_t *row_status, void *workspace, size_t workspace_bytes,
+                              aces_stream_t stream) {
     if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
     if (workspace_bytes < aces_workspace_bytes(B, K, V, k)) return ACES_ERR_INVALID_ARG;
     return verify_impl(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
@@ -208,11 +201,10 @@ aces_status aces_sparsify(const void *target_logits, aces_dtype dt, int rows, in
     a.topk_probs = topk_probs;
     a.tail = tail_mass;
     a.row_status = row_status;
-    a.ws = ws_carve(workspace, rows, rows, 0, false, true, V);
+    a.ws = ws_carve(workspace, rows, rows, 0, false);
     a.accept_len = nullptr;
     a.out_token = nullptr;
-    a.ng = 0;
-    return run_rows(a, dt, reinterpret_cast<cudaStream_t>(stream));
+    return run_rows(a, dt, false, reinterpret_cast<cudaStream_t>(stream));
 }
 
 static aces_status fill_cache_args(CacheArgs &c, const int32_t *F_host, int B, int K, int V) {
@@ -301,7 +293,7 @@ aces_status aces_cloud_step(const void *target_logits, aces_dtype dt, const floa
                             size_t workspace_bytes, aces_stream_t stream) {
     aces_status st = verify_check(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
                                   accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status,
-                                  workspace, workspace_bytes, true, true);
+                                  workspace, workspace_bytes, true);
     if (st != ACES_OK) return st;
     if (workspace_bytes < aces_workspace_bytes(B, K, V, k)) return ACES_ERR_INVALID_ARG;
     CacheArgs c;
@@ -318,7 +310,7 @@ aces_status aces_cloud_step(const void *target_logits, aces_dtype dt, const floa
     const aces_status sc = cache_launch(c, ss->s);
     const aces_status sv = verify_impl(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
                                        accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status,
-                                       workspace, workspace_bytes, true, true, stream);
+                                       workspace, workspace_bytes, true, false, stream);
     // join: later work on `stream` waits for the cache build (also after a failure)
     if (cudaEventRecord(ss->join, ss->s) != cudaSuccess || cudaStreamWaitEvent(s, ss->join, 0) != cudaSuccess)
         return ACES_ERR_CUDA;
@@ -423,3 +415,27 @@ const char *aces_status_string(aces_status s) {
 }
 
 }  // extern "C"
+
+#ifdef ACES_CHECKED
+// The first out-of-range index met by any kernel since the last call (see
+// ACES_IN in common.cuh): out = {site, index, bound}, site 0 when none.
+// Waits for the device.  Clears every word.
+extern "C" aces_status aces_checked_violation(unsigned long long out[3]) {
+    if (!out) return ACES_ERR_INVALID_ARG;
+    if (cudaDeviceSynchronize() != cudaSuccess) return ACES_ERR_CUDA;
+    cudaError_t (*take[])(unsigned long long *) = {check_take_rows_cap, check_take_rows_general, check_take_resolve,
+                                                   check_take_cache, check_take_resample, check_take_kv,
+                                                   check_take_mask};
+    out[0] = out[1] = out[2] = 0ull;
+    for (auto f : take) {
+        unsigned long long w[3];
+        if (f(w) != cudaSuccess) return ACES_ERR_CUDA;
+        if (out[0] == 0ull && w[0] != 0ull) {
+            out[0] = w[0];
+            out[1] = w[1];
+            out[2] = w[2];
+        }
+    }
+    return ACES_OK;
+}
+#endif

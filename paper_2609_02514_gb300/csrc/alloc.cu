@@ -12,6 +12,7 @@
 #include <cmath>
 #include <vector>
 
+#define ACES_FILE 2  // site numbers of the checked build
 #include "common.cuh"
 
 extern "C" {

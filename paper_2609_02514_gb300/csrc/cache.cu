@@ -7,10 +7,16 @@
 //                   One HBM pass keeps a sorted top-TOPL list per thread
 //                   (TOPL = 4 when every F_d <= 4, else 8), filtered by one
 //                   integer max and compare per four values against the raw
-//                   bits of the list's last entry; the block then extracts
-//                   maxima one at a time.  Fan-outs above TOPL repeat the
-//                   pass below the last extracted order value.
+//                   bits of the list's last entry.  F_d <= TOPL: the block
+//                   extracts maxima one at a time.  F_d > TOPL: the 2048
+//                   entries of all lists are sorted in shared memory; every
+//                   id a thread dropped lies below its full list's last
+//                   entry, so when the largest such entry is below the
+//                   F_d-th sorted entry, the first F_d are the answer (one
+//                   pass).  Otherwise the pass is repeated below the last
+//                   extracted order value, TOPL maxima at a time.
 //   k_cache_lookup  one thread per sequence scanning the F_pi branches.
+#define ACES_FILE 3  // site numbers of the checked build
 #include "common.cuh"
 
 namespace aces {
@@ -36,6 +42,9 @@ __device__ __forceinline__ void list_insert(unsigned long long (&Lst)[TOPL], uns
 template <bool VEC, int TOPL>
 __global__ void __launch_bounds__(NTC, 4) k_cache_build(CacheArgs a) {
     __shared__ unsigned long long redu[NTC / 32];
+    // the union of the per-thread lists (fan-outs above TOPL)
+    __shared__ unsigned long long uni[TOPL == 8 ? NTC * TOPL : 1];
+    __shared__ int s_done;
     const int row = blockIdx.x, tid = threadIdx.x;
     const int b = row / a.K, d = row % a.K;
     const int Fd = a.F[d];
@@ -92,6 +101,32 @@ __global__ void __launch_bounds__(NTC, 4) k_cache_build(CacheArgs a) {
                 for (int x = tid; x < a.V; x += NTC) {
                     const float qv = __ldg(qr + x);
                     if (__float_as_uint(qv) >= thr) consider(qv, x);
+                }
+            }
+            if (TOPL == 8 && Fd > TOPL && got == 0 && ub == ~0ull) {
+                // one pass for the whole fan-out when the union of the lists
+                // provably holds the Fd largest
+                const unsigned long long bound = Lst[TOPL - 1];  // 0: nothing dropped
+                const unsigned long long D = block_reduce_n<NTC>(bound, redu, MaxU64());
+#pragma unroll
+                for (int i = 0; i < TOPL; ++i) uni[tid * TOPL + i] = Lst[i];
+                __syncthreads();
+                bitonic_sort_desc(uni, NTC * TOPL);
+                const unsigned long long vF = ACES_IN(Fd - 1, NTC * TOPL) ? uni[Fd - 1] : ~0ull;
+                if (tid == 0) s_done = D == 0ull || D < vF;
+                __syncthreads();
+                if (s_done) {
+                    int n = 0;  // positive entries among the first Fd
+                    for (int j = tid; j < Fd; j += NTC) {
+                        const unsigned long long o = uni[j];
+                        if (o != 0ull) {
+                            bt[j] = (int32_t)order_id(o);
+                            bp[j] = order_value(o) / den;
+                            ++n;
+                        }
+                    }
+                    got = (int)block_reduce_n<NTC>((unsigned long long)n, redu, SumU64());
+                    break;
                 }
             }
             const int take = min(TOPL, Fd - got);
@@ -164,5 +199,9 @@ cudaError_t launch_cache_lookup(const int32_t *bt, const CacheArgs &a, const int
     k_cache_lookup<<<(a.B + 255) / 256, 256, 0, s>>>(bt, a, accept_len, token, slot);
     return cudaGetLastError();
 }
+
+#ifdef ACES_CHECKED
+cudaError_t check_take_cache(unsigned long long out[3]) { return check_take(out); }
+#endif
 
 }  // namespace aces

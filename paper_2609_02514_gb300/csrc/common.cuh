@@ -8,10 +8,52 @@
 
 namespace aces {
 
-constexpr int NT = 512;             // threads per CTA for every row kernel
+// ---------------------------------------------------------------------------
+// Checked build (compiled with -DACES_CHECKED, for tests).  ACES_IN(i, n) is
+// true when 0 <= i < n; otherwise it records the first violation met in this
+// translation unit -- the site (file number * 10000 + line), the index and
+// the bound -- in a device word, and the caller skips the access (a store)
+// or reads nothing (a load).  Nothing traps.  In the normal build it is the
+// constant true and costs nothing.  Each .cu file defines ACES_FILE (its
+// number) before including this header.
+#ifndef ACES_FILE
+#define ACES_FILE 0
+#endif
+#ifdef ACES_CHECKED
+static __device__ unsigned long long g_check[3];  // site (0: none), index, bound
+static __device__ __noinline__ bool check_fail(long long i, long long n, int site) {
+    if (atomicCAS(&g_check[0], 0ull, (unsigned long long)site) == 0ull) {
+        g_check[1] = (unsigned long long)i;
+        g_check[2] = (unsigned long long)n;
+        __threadfence();
+    }
+    return false;
+}
+#define ACES_IN(i, n)                                                              \
+    ((unsigned long long)(long long)(i) < (unsigned long long)(long long)(n)       \
+         ? true                                                                    \
+         : ::aces::check_fail((long long)(i), (long long)(n), ACES_FILE * 10000 + __LINE__))
+// reads this translation unit's word into out[3] and clears it
+static inline cudaError_t check_take(unsigned long long out[3]) {
+    cudaError_t e = cudaMemcpyFromSymbol(out, g_check, sizeof(g_check));
+    if (e != cudaSuccess) return e;
+    const unsigned long long z[3] = {0ull, 0ull, 0ull};
+    return cudaMemcpyToSymbol(g_check, z, sizeof(z));
+}
+cudaError_t check_take_rows_cap(unsigned long long out[3]);
+cudaError_t check_take_rows_general(unsigned long long out[3]);
+cudaError_t check_take_resolve(unsigned long long out[3]);
+cudaError_t check_take_cache(unsigned long long out[3]);
+cudaError_t check_take_resample(unsigned long long out[3]);
+cudaError_t check_take_kv(unsigned long long out[3]);
+cudaError_t check_take_mask(unsigned long long out[3]);
+#else
+#define ACES_IN(i, n) true
+#endif
+
+constexpr int NT = 512;             // threads per CTA for the general row kernel
 constexpr int NWARP = NT / 32;
-constexpr int SKETCH_CAP = 16384;   // max sketch groups per row (fast path)
-constexpr int NBIN = 256;           // sketch bins of width T/8 below the max
+constexpr int NBIN = 256;           // bins of width T/8 below the row max
 constexpr int BIN_PER_T = 8;
 
 // Row-level flags kept in the workspace.
@@ -20,6 +62,12 @@ constexpr int RS_NONFINITE = 2;
 // handed to the general kernel: kref holds the row max, c the log2 reference
 // of the row's exp-sum and S_nuc that exp-sum
 constexpr int RS_HANDOFF = 4;
+// the nucleus ends among the ids of one bfloat16 value whose ids were not
+// kept: cut holds that value's 32-bit order key in its high word and j, the
+// number of its ids (in id order) inside the nucleus, in its low word; the
+// resolve step turns it into the order value of the last nucleus id before
+// it reads the row
+constexpr int RS_LAZY = 8;
 
 // Per-row state written by the row kernels and read by the resolve kernel.
 struct RowStat {
@@ -306,87 +354,66 @@ struct SegSum {
 constexpr int NSEG_MAX = 16;
 constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual step
 
-constexpr int WS_COUNTERS = 32;  // bytes of path counters at the start of the workspace
+constexpr int WS_COUNTERS = 256;  // bytes of path counters and depth hints at the start of the workspace
+constexpr int WS_DEPTH0 = 16;     // first of the 40 depth-histogram counters (int index)
 // Workspace layout (all offsets 16-byte aligned)
 struct Workspace {
-    int *fb_count;             // [8]   [0] rows handed to the general path, [1] reserved (no
-                               //       kernel waits on another),
-                               //       [2] rows certified by the full sketch, [3] rows ordered by
-                               //       bitonic sort, [4] rows the general path finished by radix
-                               //       selection, [5] rows split over several CTAs, [6] rows
-                               //       the general path finished by value histogram (path
-                               //       counters, cleared by every call)
+    int *fb_count;             // [64]  path counters and depth hints, cleared by every call: [0] rows handed to the
+                               //       general kernel, [1] reserved (no kernel waits on another),
+                               //       [2] rows captured by value histogram, [3] rows ordered by
+                               //       bitonic sort, [4] rows the general kernel finished by radix
+                               //       selection, [5] rows whose cut was left to the resolve step,
+                               //       [6] rows the general kernel finished by value histogram,
+                               //       [7] accept tests that ranked the draft token among ties,
+                               //       [8] rows that published the depth they needed,
+                               //       [16..55] how many rows needed each depth (the deeper of
+                               //       their crossing and payload end, in sample bins of T/4
+                               //       below the row's sample max)
     RowStat *stats;            // [rows]
     int *acc;                  // [B*K] accept bits
     int *fb_list;              // [rows]
     SegSum *seg;               // [B*NSEG_MAX]     (verify only)
-    int *seqcnt;               // [B]              (verify only) rows of the sequence finished by the fast kernel
+    int *seqcnt;               // [B]              (verify only) rows of the sequence finished by the row kernel
     int *seqdone;              // [B]              (verify only) token already drawn
+    int *cutcnt;               // [B]              (verify only) segments that counted their ties
+    int *tiecnt;               // [B*NSEG_MAX]     (verify only) ties of the cut value per segment
     unsigned long long *nuc;   // [rows*NUC_CAP]   (verify with lists) nucleus order values
-    int *rowcnt;               // [SPLIT_ROWS_MAX] (split rows) parts finished
-    unsigned char *parts;      // [SPLIT_ROWS_MAX * split_row_bytes(V)] (split rows) partial results
-    size_t part_stride;        // split_row_bytes(V)
 };
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
 // rows = B*(K+1) target rows; nseq = B sequences with K draft positions (K = 0: sparsify);
 // lists: keep every row's nucleus (up to NUC_CAP ids) for the residual step
-// Rows split over several CTAs (the last partial wave of a large batch, or
-// every row of a small one): at most SPLIT_ROWS_MAX rows per call, in at most
-// SPLIT_P_MAX parts of SPLIT_NT threads.  Per split row the workspace keeps
-// each part's statistics and top group maxima, and the row's sketch.
-constexpr int SPLIT_ROWS_MAX = 640;
-constexpr int SPLIT_P_MAX = 4;
-constexpr int SPLIT_NT = 256;
-struct PartStat {
-    float m, kref;  // the part's max and reference
-    double S;       // its exp-sum against kref
-};
-__host__ __device__ inline size_t split_row_bytes(int V) {
-    // sketch: at most V / 16 + 1 groups of 4 bytes (float32 rows, four chunks per group)
-    return align16((size_t)SPLIT_P_MAX * sizeof(PartStat) + (size_t)SPLIT_P_MAX * 2 * SPLIT_NT * 4 +
-                   ((size_t)V / 16 + 1) * 4);
-}
-__host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K, bool lists, bool split = false,
-                                           int V = 0) {
+__host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K, bool lists) {
     size_t b = WS_COUNTERS + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
                align16((size_t)rows * 4);
     if (K > 0) {
-        b += 2 * align16((size_t)nseq * 4) + align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
+        b += 3 * align16((size_t)nseq * 4) + align16((size_t)nseq * NSEG_MAX * sizeof(SegSum)) +
+             align16((size_t)nseq * NSEG_MAX * 4);
         if (lists) b += (size_t)rows * NUC_CAP * 8;
-    }
-    if (split) {
-        const int sr = rows < SPLIT_ROWS_MAX ? rows : SPLIT_ROWS_MAX;
-        b += align16((size_t)SPLIT_ROWS_MAX * 4) + (size_t)sr * split_row_bytes(V);
     }
     return b;
 }
-// bytes at the start of the workspace that every call clears: the counters,
-// for verification the per-sequence row counts and done flags, and the
-// split rows' part counts
-__host__ __device__ inline size_t ws_clear_bytes(int nseq, int K, bool split = false) {
-    return WS_COUNTERS + (K > 0 ? 2 * align16((size_t)nseq * 4) : 0) +
-           (split ? align16((size_t)SPLIT_ROWS_MAX * 4) : 0);
+// bytes at the start of the workspace that every call clears: the counters
+// and, for verification, the per-sequence row counts, done flags and
+// segment counts
+__host__ __device__ inline size_t ws_clear_bytes(int nseq, int K) {
+    return WS_COUNTERS + (K > 0 ? 3 * align16((size_t)nseq * 4) : 0);
 }
-__host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K, bool lists,
-                                             bool split = false, int V = 0) {
+__host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K, bool lists) {
     char *p = (char *)base;
     Workspace w;
     w.fb_count = (int *)p;
     p += WS_COUNTERS;
     w.seqcnt = nullptr;
     w.seqdone = nullptr;
+    w.cutcnt = nullptr;
+    w.tiecnt = nullptr;
     if (K > 0) {
         w.seqcnt = (int *)p;
         p += align16((size_t)nseq * 4);
         w.seqdone = (int *)p;
         p += align16((size_t)nseq * 4);
-    }
-    w.rowcnt = nullptr;
-    w.parts = nullptr;
-    w.part_stride = split_row_bytes(V);
-    if (split) {
-        w.rowcnt = (int *)p;
-        p += align16((size_t)SPLIT_ROWS_MAX * 4);
+        w.cutcnt = (int *)p;
+        p += align16((size_t)nseq * 4);
     }
     w.stats = (RowStat *)p;
     p += align16((size_t)rows * sizeof(RowStat));
@@ -399,12 +426,13 @@ __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, in
     if (K > 0) {
         w.seg = (SegSum *)p;
         p += align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
+        w.tiecnt = (int *)p;
+        p += align16((size_t)nseq * NSEG_MAX * 4);
         if (lists) {
             w.nuc = (unsigned long long *)p;
             p += (size_t)rows * NUC_CAP * 8;
         }
     }
-    if (split) w.parts = (unsigned char *)p;
     return w;
 }
 
@@ -424,10 +452,16 @@ struct RowArgs {
     int32_t *accept_len;   // verification outputs (null for sparsify)
     int32_t *out_token;
     Workspace ws;
-    int ng;                // sketch groups per row
-    int r_full;            // rows r < r_full take one CTA each; the rest are split
-    int P;                 // parts of a split row (1: none)
-    int gper;              // sketch groups per part
+    // capture row kernel (16-byte aligned rows): the row's 16-byte chunks are
+    // read in tiles of 32 (one coalesced warp load), tile t of the row order
+    // at position (t * pstride) mod ntile, so that the first iteration reads
+    // a strided sample of samp_frac of the row
+    int ntile, pstride, pstride_w, pstride_it;
+    int it_partial;        // iteration that reads the row's partial last tile (-1: none)
+    float samp_frac;
+    float inv_ws;          // sample bins per unit of logit: SPB / T
+    int nmin, npay;        // ids the capture must reach: for the nucleus and payload, for the payload list
+    int force_fb;          // hand every row to the general kernel (the library's exact reference path)
 };
 
 // Arguments of the sequence kernel.
@@ -504,7 +538,7 @@ __device__ void draw_from_list(const Workspace &ws, const float *q, const float 
         return;
     }
     if (rs.nnuc < 0) return;  // no list: the scan kernels draw this sequence
-    const int n = rs.nnuc;
+    const int n = ACES_IN(rs.nnuc - 1, NUC_CAP) ? rs.nnuc : 0;
     const unsigned long long *lst = ws.nuc + (size_t)r * NUC_CAP;
     const float *qrow = pi < K ? q + ((size_t)b * K + pi) * V : nullptr;
     const float inv_S = inv_mass(rs.S_nuc);
@@ -513,7 +547,7 @@ __device__ void draw_from_list(const Workspace &ws, const float *q, const float 
         const uint32_t id = order_id(o);
         const float p = ex2(fmaf(order_value(o), rs.c, -rs.kref)) * inv_S;
         float rr = p;
-        if (qrow) {
+        if (qrow && ACES_IN(id, V)) {
             const float qx = __ldg(qrow + id);
             if (!(qx >= 0.0f)) sh->bad = 1;
             rr = fmaxf(p - qx, 0.0f);
@@ -537,13 +571,15 @@ __device__ void draw_from_list(const Workspace &ws, const float *q, const float 
         int rank = 0;
 #pragma unroll 4
         for (int j = 0; j < n; ++j) rank += skey[j] < key;
-        srt[rank] = key;
+        if (ACES_IN(rank, NUC_CAP)) srt[rank] = key;
     }
     __syncthreads();
     // two consecutive entries (in id order) per thread
     const int e0 = 2 * tid, e1 = 2 * tid + 1;
-    const int i0 = e0 < n ? (int)(srt[e0] & 0xFFFFFFFFull) : -1;
-    const int i1 = e1 < n ? (int)(srt[e1] & 0xFFFFFFFFull) : -1;
+    int i0 = e0 < n ? (int)(srt[e0] & 0xFFFFFFFFull) : -1;
+    int i1 = e1 < n ? (int)(srt[e1] & 0xFFFFFFFFull) : -1;
+    if (i0 >= 0 && !ACES_IN(i0, NUC_CAP)) i0 = -1;
+    if (i1 >= 0 && !ACES_IN(i1, NUC_CAP)) i1 = -1;
     const unsigned long long r0 = i0 >= 0 ? rfx[i0] : 0ull, r1 = i1 >= 0 ? rfx[i1] : 0ull;
     const unsigned long long R = block_reduce_n<NTH>(r0 + r1, red, SumU64());
     const int mode = R == 0ull;  // p <= q everywhere: draw from p itself
@@ -593,22 +629,20 @@ __device__ void nonfinite_row(const RowArgs &a, int r) {
 }
 
 // host launchers (defined next to their kernels)
-size_t rows_fast_smem(int dt, int gc, int nch);
-int rows_fast_gc(int dt, int V);
-cudaError_t launch_rows_fast(const RowArgs &a, int dt, int gc, size_t smem, cudaStream_t s);
-int rows_fast_per_sm(int dt, int gc, size_t smem);
+void rows_cap_layout(RowArgs &a, int dt);
+cudaError_t launch_rows_cap(const RowArgs &a, int dt, cudaStream_t s);
 cudaError_t launch_rows_general(const RowArgs &a, int dt, bool vec, int direct, int grid, cudaStream_t s);
 cudaError_t launch_resolve(const ResolveArgs &a, int dt, bool vec, cudaStream_t s);
 // aces_verify with two choices, neither of which changes the results: lists =
-// false keeps no nucleus lists (the residual draw scans its row), split =
-// false never splits a row over CTAs; the call then needs
-// ws_bytes(rows, B, K, lists, split, V) bytes of workspace.
+// false keeps no nucleus lists (the residual draw scans its row; the call then
+// needs ws_bytes(rows, B, K, lists) bytes of workspace), exact = true hands
+// every row to the general kernel.
 aces_status verify_impl(const void *target_logits, aces_dtype dt, const float *draft_probs,
                         const int32_t *draft_tokens, const float *uniforms, int B, int K, int V,
                         float T, float top_p, int32_t *accept_len, int32_t *out_token, int k,
                         int32_t *topk_ids, float *topk_probs, float *tail_mass,
                         int32_t *row_status, void *workspace, size_t workspace_bytes, bool lists,
-                        bool split, aces_stream_t stream);
+                        bool exact, aces_stream_t stream);
 cudaError_t launch_cache_build(const CacheArgs &a, bool vec, cudaStream_t s);
 cudaError_t launch_tree_mask(const int *off, int K, int branch_len, int n, int words, uint32_t *mask,
                              int32_t *depth, cudaStream_t s);

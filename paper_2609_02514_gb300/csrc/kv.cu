@@ -10,6 +10,7 @@
 // overlap (the source always lies above the destination), so each warp
 // moves them in increasing order, in rounds no longer than the distance
 // between the two, loading a whole round before storing it.
+#define ACES_FILE 4  // site numbers of the checked build
 #include "common.cuh"
 
 namespace aces {
@@ -51,6 +52,7 @@ __global__ void __launch_bounds__(NTK) k_compact_kv(KvArgs a) {
     const long long dst = (long long)t + pi;
     if (src == dst) return;
     char *base = a.kv + (((size_t)plane * a.B + b) * a.H + h) * (size_t)a.S * a.row_bytes;
+    if (!ACES_IN(src + L - 1, a.S) || !ACES_IN(dst, a.S)) return;
     const char *from = base + (size_t)src * a.row_bytes;
     char *to = base + (size_t)dst * a.row_bytes;
     const size_t total = (size_t)L * a.row_bytes;
@@ -96,5 +98,9 @@ cudaError_t launch_compact_kv(void *kv, int planes, int B, int H, int S, size_t 
     k_compact_kv<<<(unsigned)grid, NTK, 0, s>>>(a);
     return cudaGetLastError();
 }
+
+#ifdef ACES_CHECKED
+cudaError_t check_take_kv(unsigned long long out[3]) { return check_take(out); }
+#endif
 
 }  // namespace aces

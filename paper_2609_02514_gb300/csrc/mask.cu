@@ -9,6 +9,7 @@
 // writes one 32-bit word of one row: a token's allowed keys are at most two
 // intervals, [0, a) of the main chain and [b, c] of its own branch, so each
 // word is two interval masks.
+#define ACES_FILE 5  // site numbers of the checked build
 #include "common.cuh"
 
 namespace aces {
@@ -66,5 +67,9 @@ cudaError_t launch_tree_mask(const int *off, int K, int branch_len, int n, int w
     k_tree_mask<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(a);
     return cudaGetLastError();
 }
+
+#ifdef ACES_CHECKED
+cudaError_t check_take_mask(unsigned long long out[3]) { return check_take(out); }
+#endif
 
 }  // namespace aces

@@ -18,6 +18,7 @@
 // and must not be issued.
 #include <mutex>
 
+#define ACES_FILE 6  // site numbers of the checked build
 #include "common.cuh"
 
 namespace {
@@ -54,19 +55,16 @@ extern "C" aces_status aces_verify_noalloc(const void *target_logits, aces_dtype
     if (B < 1 || K < 1 || K > ACES_MAX_K) return ACES_ERR_INVALID_ARG;
     const size_t full = aces_workspace_bytes(B, K, V, k);
     if (full == 0) return ACES_ERR_INVALID_ARG;
-    // The nucleus lists (4 KiB per row) fit for small batches only, the
-    // split-row areas (about V / 4 bytes per row) for a few rows of a small
-    // vocabulary; without either the call needs ws_bytes(rows, B, K, false)
-    // bytes.
+    // The nucleus lists (4 KiB per row) fit for small batches only; without
+    // them the call needs ws_bytes(rows, B, K, false) bytes.
     const int rows = B * (K + 1);
     const size_t cap = (size_t)ACES_NOALLOC_SCRATCH_BYTES;
-    const bool split = full <= cap;
-    const bool lists = aces::ws_bytes(rows, B, K, true) <= cap;
+    const bool lists = full <= cap;
     if (aces::ws_bytes(rows, B, K, false) > cap) return ACES_ERR_UNSUPPORTED;  // batch too large
     void *scratch = nullptr;
     const aces_status st = scratch_address(&scratch);
     if (st != ACES_OK) return st;
     return aces::verify_impl(target_logits, dt, draft_probs, draft_tokens, uniforms, B, K, V, T, top_p,
                              accept_len, out_token, k, topk_ids, topk_probs, tail_mass, row_status, scratch,
-                             cap, lists, split, stream);
+                             cap, lists, false, stream);
 }

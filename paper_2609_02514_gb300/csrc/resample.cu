@@ -24,6 +24,7 @@
 //      every weight an integer in units of 2^-52 (exact, order independent).
 #include <cooperative_groups.h>
 
+#define ACES_FILE 7  // site numbers of the checked build
 #include "common.cuh"
 
 namespace aces {
@@ -143,8 +144,10 @@ __global__ void __cluster_dims__(SCL, 1, 1) __launch_bounds__(NTS) k_resample_sp
         if (key == ~0ull) continue;
         int rank = 0;
         for (int i = 0; i < a.k; ++i) rank += skey[i] < key;
-        sid[rank] = (int)(key >> 32);
-        sidx[rank] = (int)(key & 0xFFFFFFFFull);
+        if (ACES_IN(rank, SPAY)) {
+            sid[rank] = (int)(key >> 32);
+            sidx[rank] = (int)(key & 0xFFFFFFFFull);
+        }
         atomicAdd(&s_n, 1);
     }
     __syncthreads();
@@ -152,7 +155,7 @@ __global__ void __cluster_dims__(SCL, 1, 1) __launch_bounds__(NTS) k_resample_sp
     for (int i = tid; i < n; i += NTS) {
         const int x = sid[i], j = sidx[i];
         float w = fmaxf(P[j], 0.0f);
-        if (qr) {
+        if (qr && ACES_IN(x, V)) {
             const float qx = __ldg(qr + x);
             if (!(qx >= 0.0f)) s_bad = 1;
             w = fmaxf(P[j] - qx, 0.0f);
@@ -415,5 +418,9 @@ cudaError_t launch_resample_sparse(const int32_t *accept_len, const int32_t *ids
     else k_resample_sparse<false><<<B * SCL, NTS, 0, s>>>(a);
     return cudaGetLastError();
 }
+
+#ifdef ACES_CHECKED
+cudaError_t check_take_resample(unsigned long long out[3]) { return check_take(out); }
+#endif
 
 }  // namespace aces

@@ -16,10 +16,17 @@
 //                   those ids only, they are ordered by id, and the draw is
 //                   taken from their prefix sums.  Identical to the scan
 //                   below, whose other terms are all zero.
+//   k_resolve_cut   (B x nseg CTAs) when row pi kept its cut as (value v,
+//                   count j) (RS_LAZY: the nucleus ends among the ids of one
+//                   bfloat16 value, which the row kernel did not list): each
+//                   CTA counts the ids of value v in its segment, the last
+//                   CTA of the sequence finds the segment holding the j-th
+//                   and scans it for that id, the exact cut
 //   k_resolve_seg   (B x nseg CTAs) every other sequence: segment sums of
 //                   the residual and of p over the whole row
 //   k_resolve_pick  (B CTAs) locates the segment holding the draw and scans
 //                   it in 2048-id tiles until the crossing id is found
+#define ACES_FILE 8  // site numbers of the checked build
 #include "common.cuh"
 
 namespace aces {
@@ -82,6 +89,99 @@ __device__ __forceinline__ void mass_fx(const char *zrow, const float *qrow, int
     }
 }
 
+
+// ids of [x0, x0 + EPT) whose logit has order key vkey (bit e of the result)
+template <int DT, bool VEC>
+__device__ __forceinline__ uint32_t ties_of(const char *zrow, int V, int x0, uint32_t vkey) {
+    using E = Elem<DT>;
+    uint32_t m = 0u;
+    if (VEC && x0 + EPT <= V) {
+        if (DT == ACES_BF16) {
+            const uint4 w = ldg16(zrow + (size_t)x0 * 2);
+#pragma unroll
+            for (int e = 0; e < EPT; ++e) m |= (uint32_t)(fkey(E::get(w, e)) == vkey) << e;
+        } else {
+            const uint4 w0 = ldg16(zrow + (size_t)x0 * 4), w1 = ldg16(zrow + (size_t)x0 * 4 + 16);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                m |= (uint32_t)(fkey(Elem<ACES_F32>::get(w0, e)) == vkey) << e;
+                m |= (uint32_t)(fkey(Elem<ACES_F32>::get(w1, e)) == vkey) << (e + 4);
+            }
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < EPT; ++e) {
+            const int x = x0 + e;
+            if (x < V) m |= (uint32_t)(fkey(E::load1(zrow, x)) == vkey) << e;
+        }
+    }
+    return m;
+}
+
+template <int DT, bool VEC>
+__global__ void __launch_bounds__(NTR) k_resolve_cut(ResolveArgs a, int nseg, int seglen) {
+    using E = Elem<DT>;
+    __shared__ int s_pi, s_last, s_seg, s_need, s_id;
+    __shared__ unsigned long long red[NTR / 32];
+    const int b = blockIdx.x / nseg, sg = blockIdx.x % nseg, tid = threadIdx.x;
+    pdl_wait();  // the row kernels are complete
+    if (a.ws.fb_count[5] == 0 || a.ws.seqdone[b]) return;  // no cut left open / token already drawn
+    if (tid == 0) s_pi = first_reject(a.ws, b, a.K);
+    __syncthreads();
+    const int r = b * (a.K + 1) + s_pi;
+    const RowStat rs = a.ws.stats[r];
+    if (!(rs.flags & RS_LAZY)) return;
+    const uint32_t vkey = (uint32_t)(rs.cut >> 32);
+    const int j = (int)(uint32_t)rs.cut;  // >= 1
+    const char *zrow = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
+    const int x_lo = sg * seglen, x_hi = min(a.V, x_lo + seglen);
+    unsigned long long cnt = 0ull;
+    for (int x0 = x_lo + tid * EPT; x0 < x_hi; x0 += TILE) cnt += __popc(ties_of<DT, VEC>(zrow, x_hi, x0, vkey));
+    const unsigned long long tot = block_reduce_n<NTR>(cnt, red, SumU64());
+    if (tid == 0) {
+        a.ws.tiecnt[(size_t)b * NSEG_MAX + sg] = (int)tot;
+        // releases the count; the last segment acquires the others'
+        s_last = atomic_add_acq_rel(&a.ws.cutcnt[b], 1) == nseg - 1;
+    }
+    __syncthreads();
+    if (!s_last) return;
+    if (tid == 0) {
+        int before = 0, seg = nseg - 1;
+        for (int t = 0; t < nseg; ++t) {
+            const int c = a.ws.tiecnt[(size_t)b * NSEG_MAX + t];
+            if (before + c >= j) {
+                seg = t;
+                break;
+            }
+            before += c;
+        }
+        s_seg = seg;
+        s_need = j - before;  // rank (1-based) of the cut among the segment's ties
+        s_id = -1;
+    }
+    __syncthreads();
+    const int y_lo = s_seg * seglen, y_hi = min(a.V, y_lo + seglen);
+    unsigned long long base = 0ull;
+    for (int t0 = y_lo; t0 < y_hi; t0 += TILE) {
+        const int x0 = t0 + tid * EPT;
+        const uint32_t m = x0 < y_hi ? ties_of<DT, VEC>(zrow, y_hi, x0, vkey) : 0u;
+        unsigned long long total;
+        const unsigned long long ex = base + block_exscan_n<NTR>((unsigned long long)__popc(m), red, &total);
+        const unsigned long long need = (unsigned long long)s_need;
+        if (ex < need && need <= ex + (unsigned long long)__popc(m) && ACES_IN(x0, y_hi)) {
+            uint32_t mm = m;
+            for (unsigned long long q = ex + 1ull; q < need; ++q) mm &= mm - 1u;
+            s_id = x0 + __ffs(mm) - 1;
+        }
+        __syncthreads();
+        if (s_id >= 0) break;
+        base += total;
+    }
+    if (tid == 0 && s_id >= 0 && ACES_IN(s_id, a.V)) {
+        a.ws.stats[r].cut = order_val(vkey, (uint32_t)s_id);
+        a.ws.stats[r].flags = rs.flags & ~RS_LAZY;
+    }
+}
 
 template <int DT, bool VEC>
 __global__ void __launch_bounds__(NTR) k_resolve_seg(ResolveArgs a, int nseg, int seglen) {
@@ -243,23 +343,32 @@ int resolve_segments(int V) {
     return nseg < 1 ? 1 : (nseg > NSEG_MAX ? NSEG_MAX : nseg);
 }
 
-// Both kernels follow the row kernels of the same call and overlap their drain.
+// The kernels follow the row kernels of the same call and overlap their drain.
 cudaError_t launch_resolve(const ResolveArgs &a, int dt, bool vec, cudaStream_t s) {
     const int nseg = resolve_segments(a.V);
     int seglen = (a.V + nseg - 1) / nseg;
     seglen = (seglen + EPT - 1) / EPT * EPT;
     const int g1 = a.B * nseg;
-    void (*seg)(ResolveArgs, int, int), (*pick)(ResolveArgs, int, int);
+    void (*seg)(ResolveArgs, int, int), (*pick)(ResolveArgs, int, int), (*cut)(ResolveArgs, int, int);
     if (dt == ACES_BF16) {
+        cut = vec ? k_resolve_cut<ACES_BF16, true> : k_resolve_cut<ACES_BF16, false>;
         seg = vec ? k_resolve_seg<ACES_BF16, true> : k_resolve_seg<ACES_BF16, false>;
         pick = vec ? k_resolve_pick<ACES_BF16, true> : k_resolve_pick<ACES_BF16, false>;
     } else {
+        cut = nullptr;  // only bfloat16 rows leave a cut open
         seg = vec ? k_resolve_seg<ACES_F32, true> : k_resolve_seg<ACES_F32, false>;
         pick = vec ? k_resolve_pick<ACES_F32, true> : k_resolve_pick<ACES_F32, false>;
     }
-    cudaError_t e = launch_after(seg, (unsigned)g1, NTR, s, a, nseg, seglen);
+    cudaError_t e = cudaSuccess;
+    if (cut) e = launch_after(cut, (unsigned)g1, NTR, s, a, nseg, seglen);
+    if (e != cudaSuccess) return e;
+    e = launch_after(seg, (unsigned)g1, NTR, s, a, nseg, seglen);
     if (e != cudaSuccess) return e;
     return launch_after(pick, (unsigned)a.B, NTR, s, a, nseg, seglen);
 }
+
+#ifdef ACES_CHECKED
+cudaError_t check_take_resolve(unsigned long long out[3]) { return check_take(out); }
+#endif
 
 }  // namespace aces

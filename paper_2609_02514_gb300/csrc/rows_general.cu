@@ -19,6 +19,7 @@
 
 #include <cuda_bf16.h>
 
+#define ACES_FILE 10  // site numbers of the checked build
 #include "common.cuh"
 
 namespace aces {
@@ -139,11 +140,11 @@ __device__ __forceinline__ void hist_add(uint32_t *cnt, unsigned long long *mass
     const int d0 = __shfl_sync(0xffffffffu, d, __ffs(act) - 1);
     if (__all_sync(0xffffffffu, !ok || d == d0)) {
         const unsigned long long ms = with_mass ? warp_sum(ok ? m : 0ull) : 0ull;
-        if ((threadIdx.x & 31) == 0) {
+        if ((threadIdx.x & 31) == 0 && ACES_IN(d0, 256)) {
             atomicAdd(&cnt[d0], (uint32_t)__popc(act));
             if (with_mass) atomicAdd(&mass[d0], ms);
         }
-    } else if (ok) {
+    } else if (ok && ACES_IN(d, 256)) {
         atomicAdd(&cnt[d], 1u);
         if (with_mass) atomicAdd(&mass[d], m);
     }
@@ -401,7 +402,7 @@ __device__ bool binned_row(const RowArgs &a, int r, const char *row, float m, fl
         int rank = 0;
 #pragma unroll 4
         for (int t = 0; t < npl; ++t) rank += bs->ps[t] > key;
-        if (rank < lp) buf[rank] = key;
+        if (rank < lp && ACES_IN(rank, ACES_MAX_TOPK)) buf[rank] = key;
     }
     // the crossing bin in order (descending order value)
     {
@@ -444,7 +445,7 @@ __device__ bool binned_row(const RowArgs &a, int r, const char *row, float m, fl
         } else {
             S_nuc = redd[0];
         }
-        cut = bs->xs[ix];
+        cut = ACES_IN(ix, GB_CAP) ? bs->xs[ix] : 0ull;
         n_nuc = (long long)bs->nbelow + ix + 1;
     } else {
         S_nuc = (double)bs->S_fx * FX_INV;
@@ -578,7 +579,7 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
                         if (WS) cs += ex2(fmaf(__uint_as_float(b << 16), a.c, -kref));  // 0 for -inf
                         if (WN) nf += b != 0xFF80u;
                         const uint32_t d = km - bkey16(b);
-                        if (d <= D) atomicAdd(&vh->cnt[d], 1u);
+                        if (d <= D && ACES_IN(d, VH_W)) atomicAdd(&vh->cnt[d], 1u);
                     }
                 }
             }
@@ -707,7 +708,7 @@ __device__ bool valhist_row(const RowArgs &a, int r, const char *row, float m, f
         int rank = 0;
 #pragma unroll 4
         for (int t = 0; t < npay; ++t) rank += vh->pay[t] > key;
-        if (rank < LL) buf[rank] = key;
+        if (rank < LL && ACES_IN(rank, ACES_MAX_TOPK)) buf[rank] = key;
     }
     const int jt = dstar >= 0 ? vh->j - 1 : -1;
     for (int i = tid; i < ntie; i += NT) {
@@ -750,6 +751,7 @@ __global__ void __launch_bounds__(NT) k_rows_general(RowArgs a, int direct) {
     const int nrows = direct ? a.rows : *a.ws.fb_count;
     for (int idx = blockIdx.x; idx < nrows; idx += gridDim.x) {
         const int r = direct ? idx : a.ws.fb_list[idx];
+        if (!ACES_IN(r, a.rows)) continue;  // (the same r in every thread)
         const char *row = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
         // a row the fast kernel handed over comes with its max and its
         // exp-sum (and is finite); the max pass runs only where the paths
@@ -860,5 +862,9 @@ cudaError_t launch_rows_general(const RowArgs &a, int dt, bool vec, int direct, 
     }
     return launch_after(fn, (unsigned)grid, NT, s, a, direct);
 }
+
+#ifdef ACES_CHECKED
+cudaError_t check_take_rows_general(unsigned long long out[3]) { return check_take(out); }
+#endif
 
 }  // namespace aces

@@ -19,9 +19,13 @@ def lib():
     return A.load()
 
 
-def declared_functions():
+def declared_functions(checked=False):
+    """Functions the header declares; those of the checked build's block
+    (#ifdef ACES_CHECKED) only when checked is set."""
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    if not checked:
+        text = re.sub(r"#ifdef ACES_CHECKED.*?#endif", "", text, flags=re.S)
     return sorted(set(re.findall(r"\b(aces_[a-z_]+)\s*\(", text)))
 
 
@@ -35,6 +39,9 @@ def test_header_declares_the_four_entry_points():
 def test_library_exports_every_declared_symbol(lib):
     for name in declared_functions():
         assert hasattr(lib, name), name
+    # the checked build's extra function is not in the product library
+    extra = set(declared_functions(checked=True)) - set(declared_functions())
+    assert extra == {"aces_checked_violation"}
 
 
 def test_workspace_sizes(lib):

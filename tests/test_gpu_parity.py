@@ -89,9 +89,9 @@ def test_small_workloads_full(A, orc, name):
 
 
 @pytest.mark.parametrize("name", ["b64_k8_v152064_bf16", "b128_k16_v128256_bf16", "b256_k16_v256000_bf16"])
-def test_full_size_sampled(A, orc, name):
+def test_full_size_all_sequences(A, orc, name):
     """Full batch on the GPU as the benchmark launches it; the oracle checks
-    sampled sequences one by one; properties are checked on every sequence."""
+    every sequence (flagged ones for validity only); properties on all."""
     w = gen.WORKLOADS[name]
     inp = gen.generate(name, workers=min(16, os.cpu_count() or 1))
     g = run_gpu(A, inp, w, w.k)
@@ -107,23 +107,18 @@ def test_full_size_sampled(A, orc, name):
     assert (p.sum(-1) <= 1 + 1e-5).all()
     np.testing.assert_allclose(g["tail_mass"], 1.0 - p.astype(np.float64).sum(-1), atol=2e-5)
     assert (g["row_status"] == 0).all()
-    # oracle on a sample of sequences
-    rng = np.random.default_rng(5)
-    seqs = sorted(set([0, B - 1] + rng.choice(B, 4, replace=False).tolist()))
-    sub = {key: inp[key][seqs] for key in ("z", "q", "xt", "u")}
-    o = orc.verify(sub["z"], sub["q"], sub["xt"], sub["u"], w.T, w.top_p, w.k)
-    gs = {key: v[seqs] for key, v in g.items()}
-    res = parity.compare_verify(sub, gs, o, w.top_p, True, w.k)
-    assert res["checked_seqs"] >= len(seqs) - 2, res
-    # branch cache on the same sample
-    qt = torch.from_numpy(inp["q"]).cuda()
-    out = A.cache_build(qt, torch.from_numpy(inp["xt"]).cuda(), w.F)
-    del qt
-    gbt = out["branch_tok"].cpu().numpy()
-    gbp = out["branch_prob"].cpu().numpy()
-    obt, obp = orc.cache_build(sub["q"], sub["xt"], w.F)
-    parity.compare_cache(gbt[seqs], gbp[seqs], obt, obp)
-    slot = A.cache_lookup(out["branch_tok"], w.F, torch.from_numpy(g["accept_len"]).cuda(),
+    # the oracle on every sequence
+    o = orc.verify(inp["z"], inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
+    res = parity.compare_verify(inp, g, o, w.top_p, True, w.k)
+    # (flagged: within the flag bands of tests/parity.py, checked for validity
+    # only; on the 128256-id rows one id carries ~1.5e-5 of the mass at the
+    # crossing, so ~14% of rows lie within 1e-6 of top_p there)
+    print(f"{name}: checked {res['checked_seqs']} of {B} sequences, flagged {res['flagged_seqs']}")
+    assert res["checked_seqs"] + res["flagged_seqs"] == B
+    assert res["checked_seqs"] >= 0.7 * B, res
+    # branch cache and lookup on the whole batch
+    gbt = check_cache(A, orc, inp, w.F)
+    slot = A.cache_lookup(torch.from_numpy(gbt).cuda(), w.F, torch.from_numpy(g["accept_len"]).cuda(),
                           torch.from_numpy(g["out_token"]).cuda()).cpu().numpy()
     np.testing.assert_array_equal(slot, orc.cache_lookup(gbt, w.F, g["accept_len"], g["out_token"]))
 

@@ -1,15 +1,18 @@
-"""Parity on inputs built to drive each branch of the fast row kernel.
+"""Parity on inputs built to drive each branch of the row kernels.
 
-The workspace's first int32 words count, per call, the rows handed to the
-exact general kernel, bounded-wait timeouts, rows certified only by the full
-sketch histogram (the top group maxima kept per thread were not enough),
-rows whose candidates were ordered by bitonic sort (more than 512), rows the
-general kernel finished by radix selection, rows split over several CTAs,
-and rows the general kernel finished by its bfloat16 value histogram.  Each
-test asserts the branch it targets was taken, then compares every output
-with the float64 oracle under the rules of tests/parity.py.
+The workspace's first eight int32 words count, per call: rows handed to the
+exact general kernel, bounded-wait timeouts (reserved), rows the single-pass
+kernel captured by value histogram, rows whose candidates were ordered by
+bitonic sort (more than 512), rows the general kernel finished by radix
+selection, rows whose nucleus cut was left to the resolve step, rows the
+general kernel finished by its bfloat16 value histogram, and accept tests
+that ranked the draft token among the ids of the crossing value.  Each test
+asserts the branch it targets was taken, then compares every output with the
+float64 oracle under the rules of tests/parity.py.  Tests of the general
+kernel's own branches call the exact entry point (every row on that kernel).
 """
 import dataclasses
+import math
 
 import numpy as np
 import pytest
@@ -21,6 +24,8 @@ pytestmark = pytest.mark.gpu
 
 torch = pytest.importorskip("torch")
 
+FALLBACK, TIMEOUTS, VALUE_MODE, BITONIC, RADIX, LAZY, GEN_VALHIST, TIE_RANK = range(8)
+
 
 @pytest.fixture(scope="module")
 def A():
@@ -31,9 +36,9 @@ def A():
     return A
 
 
-def _run(A, orc, w, z):
-    """Verify the generator's q, x~, u with the logits z on both sides."""
-    inp = gen.generate(w)
+def _run(A, orc, w, z, exact=False, inp=None):
+    """Verify the generator's q, x~, u (or inp's) with the logits z on both sides."""
+    inp = dict(gen.generate(w)) if inp is None else inp
     inp["z"] = z
     if z.dtype == np.uint16:
         zt = torch.from_numpy(z.view(np.int16)).cuda().view(torch.bfloat16)
@@ -41,105 +46,209 @@ def _run(A, orc, w, z):
         zt = torch.from_numpy(z).cuda()
     q, xt, u = (torch.from_numpy(inp[key]).cuda() for key in ("q", "xt", "u"))
     ws = torch.zeros(A.workspace_bytes(w.B, w.K, w.V, w.k), dtype=torch.uint8, device="cuda")
-    g = A.verify(zt, q, xt, u, w.T, w.top_p, w.k, workspace=ws)
+    g = A.verify(zt, q, xt, u, w.T, w.top_p, w.k, workspace=ws, exact=exact)
     torch.cuda.synchronize()
     g = {key: v.cpu().numpy() for key, v in g.items()}
-    counters = ws[:28].view(torch.int32).cpu().numpy().tolist()
+    counters = ws[:32].view(torch.int32).cpu().numpy().tolist()
     o = orc.verify(z, inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
     res = parity.compare_verify(inp, g, o, w.top_p, z.dtype == np.uint16, w.k)
     return counters, res
-
-
-def _plateau(B, K, V, n_hot, group, seed):
-    """-30 everywhere except n_hot ids, one per sketch group, near 0."""
-    rng = np.random.default_rng(seed)
-    z = np.full((B, K + 1, V), -30.0, np.float32)
-    j = np.arange(n_hot)
-    ids = j * group + (j % group)
-    for b in range(B):
-        for i in range(K + 1):
-            z[b, i, ids] = rng.uniform(0.0, 1.5, n_hot).astype(np.float32)
-    return z
-
-
-def test_second_tier_certification_and_bitonic_order(A, orc):
-    # 1500 near-equal ids in 1500 different sketch groups (16 float32 logits
-    # each): the 512 per-thread top maxima carry too little mass, the full
-    # sketch certifies, and the nucleus (~1200 ids) is ordered by bitonic sort
-    w = gen.make_workload(2, 2, 32000, "f32", T=1.0, top_p=0.8, k=64, seed=31)
-    counters, res = _run(A, orc, w, _plateau(2, 2, 32000, 1500, 16, 31))
-    fallback, timeouts, second_tier, bitonic, radix, split, valhist = counters
-    assert fallback == 0 and timeouts == 0
-    # a row split over CTAs bins every part's top maxima, which here covers
-    # every hot group: the first tier then suffices
-    assert second_tier == 6 - split and bitonic == 6, counters
-    assert res["checked_seqs"] == 2
-
-
-def test_more_candidates_than_capacity_falls_back(A, orc):
-    # 3000 near-equal ids: the nucleus alone exceeds the 2048 candidates the
-    # fast kernel holds, so every row goes to the exact general kernel
-    w = gen.make_workload(2, 1, 64000, "f32", T=1.0, top_p=0.8, k=32, seed=32)
-    counters, res = _run(A, orc, w, _plateau(2, 1, 64000, 3000, 16, 32))
-    assert counters[0] == 4, counters
-    assert res["checked_seqs"] == 2
-
-
-def test_first_tier_suffices_on_the_benchmark_rows(A, orc):
-    # the first 4 sequences of the 256000-id benchmark workload (68 rows):
-    # nearly every row is certified by the per-thread top maxima, and all
-    # are ranked directly on the fast path
-    w = dataclasses.replace(gen.WORKLOADS["b256_k16_v256000_bf16"], B=4)
-    z = gen.generate(w)["z"]
-    counters, res = _run(A, orc, w, z)
-    fallback, timeouts, second_tier, bitonic = counters[:4]
-    assert fallback == 0 and timeouts == 0 and bitonic == 0, counters
-    assert second_tier <= 3, counters
-    assert res["checked_seqs"] >= 3
-
-
-@pytest.mark.parametrize("dtype,V", [("bf16", 600000), ("f32", 300000), ("f32", 600000)],
-                         ids=["bf16_gc8", "f32_gc8", "f32_general"])
-def test_large_vocabularies(A, orc, dtype, V):
-    # bf16 at 600000 ids and f32 at 300000 use 8 chunks per sketch group;
-    # f32 at 600000 exceeds the sketch and runs on the general kernel
-    w = gen.make_workload(1, 1, V, dtype, T=0.8, top_p=0.9, k=48, seed=34)
-    z = gen.generate(w)["z"]
-    counters, res = _run(A, orc, w, z)
-    assert counters[1] == 0
-    assert res["checked_seqs"] == 1
 
 
 def _bf16(z):
     return gen.f32_to_bf16(np.ascontiguousarray(z, dtype=np.float32))
 
 
-def test_value_histogram_takes_large_nucleus_bf16_rows(A, orc):
-    # rows of the 128256-id recipe (nuclei of thousands of ids): the sketch
-    # cannot order them, and the general kernel finishes every one by counting
-    # ids per bf16 value (the crossing lies among the 4096 values below the max)
-    w = gen.make_workload(2, 2, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=41)
+def _sampled_ids(V, dtype):
+    """Ids the single-pass kernel reads in its first iteration: tiles of 32
+    16-byte chunks, tile t of the row order at (t * p) mod ntile, p the
+    smallest integer >= ntile / 64 coprime with ntile, t < 64."""
+    epc = 8 if dtype == "bf16" else 4
+    ntile = -(-(V // epc) // 32)
+    p = max(1, ntile // 64)
+    while math.gcd(p, ntile) != 1:
+        p += 1
+    ids = []
+    for t in range(min(64, ntile)):
+        tile = t * p % ntile
+        ids.append(np.arange(tile * 32 * epc, min((tile + 1) * 32 * epc, V)))
+    return np.concatenate(ids)
+
+
+# ---------------------------------------------------------------------------
+# the single-pass kernel
+
+
+def test_list_mode_on_the_benchmark_rows(A, orc):
+    # the first 4 sequences of the 256000-id benchmark workload (68 rows, all
+    # estimated from their own sample): small nuclei, listed on chip; a row
+    # whose sample misleads goes to the exact kernel, which is rare
+    w = dataclasses.replace(gen.WORKLOADS["b256_k16_v256000_bf16"], B=4)
     z = gen.generate(w)["z"]
     counters, res = _run(A, orc, w, z)
-    fallback, radix, valhist = counters[0], counters[4], counters[6]
-    assert fallback >= 1 and valhist == fallback and radix == 0, counters
+    assert counters[TIMEOUTS] == 0 and counters[VALUE_MODE] == 0 and counters[LAZY] == 0, counters
+    assert counters[FALLBACK] <= 4, counters
+    assert res["checked_seqs"] >= 3
+
+
+def test_value_mode_on_large_nuclei(A, orc):
+    # rows of the 128256-id recipe (nuclei of thousands of ids): counted per
+    # bf16 value while streaming; the crossing value's ids are not listed, so
+    # the cut is left to the resolve step, which finds it for the drawn rows
+    w = gen.make_workload(3, 4, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=41)
+    z = gen.generate(w)["z"]
+    counters, res = _run(A, orc, w, z)
+    assert counters[FALLBACK] == 0 and counters[VALUE_MODE] == 15 and counters[LAZY] == 15, counters
+    assert res["checked_seqs"] >= 2
+
+
+def test_value_mode_with_listed_crossing(A, orc):
+    # 50 dominant ids at 15 outside the sampled tiles, 60000 ids in [6, 8]:
+    # the sample sees only the bulk, so the capture is deep and counted per
+    # value; the nucleus is the 50 ids, inside the payload list (the 256 ids
+    # the count floor keeps), so the cut is exact on chip
+    V = 65536
+    w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.5, k=64, seed=45)
+    rng = np.random.default_rng(45)
+    samp = _sampled_ids(V, "bf16")
+    rest = np.setdiff1d(np.arange(V), samp)
+    z = np.full((2, 2, V), -30.0, np.float32)
+    for b in range(2):
+        for i in range(2):
+            z[b, i, rng.choice(V, 60000, replace=False)] = rng.uniform(6.0, 8.0, 60000)
+            z[b, i, rng.choice(rest, 50, replace=False)] = 15.0
+    counters, res = _run(A, orc, w, _bf16(z))
+    assert counters[FALLBACK] == 0 and counters[VALUE_MODE] == 4 and counters[LAZY] == 0, counters
     assert res["checked_seqs"] >= 1
 
 
-def test_value_histogram_declines_a_crossing_below_its_window(A, orc):
+def test_value_mode_draft_token_on_the_crossing_value(A, orc):
+    # the draft token of every draft row is moved to an id holding that row's
+    # crossing value (the n_nuc-th id in order), with q > 0 there: the accept
+    # test ranks it among the ids of that value, which were not listed
+    w = gen.make_workload(2, 3, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=46)
+    inp = dict(gen.generate(w))
+    z = inp["z"]
+    zf = gen.bf16_to_f32(z).astype(np.float64)
+    o = orc.verify(z, inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
+    xt = inp["xt"].copy()
+    q = inp["q"].copy()
+    for b in range(w.B):
+        for i in range(w.K):
+            row = zf[b, i]
+            order = np.lexsort((np.arange(w.V), -row))
+            v = row[order[o["n_nuc"][b, i] - 1]]
+            same = np.flatnonzero(row == v)
+            x = int(same[len(same) // 2])  # one in the middle: in or out of the nucleus
+            xt[b, i] = x
+            if q[b, i, x] <= 0.0:
+                q[b, i, x] = 1e-3
+    inp["xt"], inp["q"] = xt, q
+    counters, res = _run(A, orc, w, z, inp=inp)
+    assert counters[TIE_RANK] >= 1 and counters[FALLBACK] == 0, counters
+    assert res["checked_seqs"] >= 1
+
+
+def test_bitonic_order_for_many_candidates(A, orc):
+    # 1500 near-equal float32 ids spread over the row, the rest far below:
+    # the list holds them all and the nucleus (~1200 ids) is ordered by
+    # bitonic sort
+    V = 32000
+    w = gen.make_workload(2, 2, V, "f32", T=1.0, top_p=0.8, k=64, seed=31)
+    rng = np.random.default_rng(31)
+    z = np.full((2, 3, V), -30.0, np.float32)
+    ids = np.arange(1500) * 21
+    z[:, :, ids] = rng.uniform(0.0, 0.5, size=(2, 3, 1500)).astype(np.float32)
+    counters, res = _run(A, orc, w, z)
+    assert counters[FALLBACK] == 0 and counters[BITONIC] == 6, counters
+    assert res["checked_seqs"] == 2
+
+
+def test_more_candidates_than_the_list_falls_back(A, orc):
+    # 3000 near-equal float32 ids: the capture exceeds the 2048-id list, so
+    # every row goes to the exact general kernel
+    V = 64000
+    w = gen.make_workload(2, 1, V, "f32", T=1.0, top_p=0.8, k=32, seed=32)
+    rng = np.random.default_rng(32)
+    z = np.full((2, 2, V), -30.0, np.float32)
+    ids = np.arange(3000) * 21
+    z[:, :, ids] = rng.uniform(0.0, 0.5, size=(2, 2, 3000)).astype(np.float32)
+    counters, res = _run(A, orc, w, z)
+    assert counters[FALLBACK] == 4, counters
+    assert res["checked_seqs"] == 2
+
+
+def test_a_misleading_sample_falls_back(A, orc):
+    # the sampled tiles hold 300 ids near 10 and nothing else; the rest of
+    # the row holds 20000 ids at 5, which carry most of the mass: the
+    # estimate puts theta far above the crossing, the capture holds too
+    # little mass, and the exact general kernel takes the row
+    V = 65536
+    w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.9, k=16, seed=47)
+    rng = np.random.default_rng(47)
+    samp = _sampled_ids(V, "bf16")
+    rest = np.setdiff1d(np.arange(V), samp)
+    z = np.full((2, 2, V), -30.0, np.float32)
+    for b in range(2):
+        for i in range(2):
+            z[b, i, rng.choice(samp, 300, replace=False)] = rng.uniform(9.8, 10.0, 300)
+            z[b, i, rng.choice(rest, 20000, replace=False)] = 5.0
+    counters, res = _run(A, orc, w, _bf16(z))
+    assert counters[FALLBACK] == 4, counters
+    assert res["checked_seqs"] >= 1
+
+
+def test_value_mode_window_exceeded_falls_back(A, orc):
+    # flat rows in [2, 3] (value mode, theta near 0.5) with one id at 1000
+    # outside the sample: it lies beyond the 1024 counted values above
+    # theta, so the row goes to the exact general kernel
+    V = 65536
+    w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.9, k=16, seed=48)
+    rng = np.random.default_rng(48)
+    samp = set(_sampled_ids(V, "bf16").tolist())
+    far = next(x for x in range(V - 1, 0, -1) if x not in samp)
+    z = rng.uniform(2.0, 3.0, size=(2, 2, V)).astype(np.float32)
+    z[:, :, far] = 1000.0
+    counters, res = _run(A, orc, w, _bf16(z))
+    assert counters[FALLBACK] == 4, counters
+    assert res["checked_seqs"] >= 1
+
+
+@pytest.mark.parametrize("dtype,V", [("bf16", 600000), ("f32", 300000), ("f32", 1 << 20)],
+                         ids=["bf16_600k", "f32_300k", "f32_1m"])
+def test_large_vocabularies(A, orc, dtype, V):
+    w = gen.make_workload(1, 1, V, dtype, T=0.8, top_p=0.9, k=48, seed=34)
+    z = gen.generate(w)["z"]
+    counters, res = _run(A, orc, w, z)
+    assert counters[TIMEOUTS] == 0
+    assert res["checked_seqs"] == 1
+
+
+# ---------------------------------------------------------------------------
+# the exact general kernel (every row handed over: aces_verify_exact)
+
+
+def test_general_value_histogram_takes_large_nucleus_bf16_rows(A, orc):
+    w = gen.make_workload(2, 2, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=41)
+    z = gen.generate(w)["z"]
+    counters, res = _run(A, orc, w, z, exact=True)
+    assert counters[FALLBACK] == 6 and counters[GEN_VALHIST] == 6 and counters[RADIX] == 0, counters
+    assert res["checked_seqs"] >= 1
+
+
+def test_general_value_histogram_declines_a_crossing_below_its_window(A, orc):
     # flat rows (T=2, top_p=0.99): the crossing lies among negative logits,
     # whose keys are below the window (below every tiny positive value); the
     # binned path takes the rows
     w = gen.make_workload(3, 2, 65536, "bf16", T=2.0, top_p=0.99, k=64, seed=41)
     z = gen.generate(w)["z"]
-    counters, res = _run(A, orc, w, z)  # (compares every unflagged output)
-    fallback, valhist = counters[0], counters[6]
-    assert fallback >= 1 and valhist == 0, counters
+    counters, res = _run(A, orc, w, z, exact=True)
+    assert counters[FALLBACK] == 9 and counters[GEN_VALHIST] == 0, counters
 
 
 @pytest.mark.parametrize("n_vals,V,expect_valhist", [(40, 32000, True), (24, 65536, False)],
                          ids=["ties_within_capacity", "ties_beyond_capacity"])
-def test_value_histogram_ties(A, orc, n_vals, V, expect_valhist):
+def test_general_value_histogram_ties(A, orc, n_vals, V, expect_valhist):
     # logits from a few distinct bf16 values: the crossing value is shared by
     # ~V/n_vals ids, taken in id order.  Up to 1024 of them the value
     # histogram orders them itself; beyond that the binned path takes the row.
@@ -147,20 +256,28 @@ def test_value_histogram_ties(A, orc, n_vals, V, expect_valhist):
     rng = np.random.default_rng(42)
     vals = np.linspace(-2.0, 2.0, n_vals).astype(np.float32)
     z = _bf16(vals[rng.integers(0, n_vals, size=(2, 3, V))])
-    counters, res = _run(A, orc, w, z)
-    fallback, valhist = counters[0], counters[6]
-    assert fallback == 6, counters
-    assert (valhist == 6) if expect_valhist else (valhist == 0), counters
+    counters, res = _run(A, orc, w, z, exact=True)
+    assert counters[FALLBACK] == 6, counters
+    assert (counters[GEN_VALHIST] == 6) if expect_valhist else (counters[GEN_VALHIST] == 0), counters
     assert res["checked_seqs"] >= 1
 
 
-def test_value_histogram_top_p_one_rows(A, orc):
-    # top_p = 1 on bf16 rows: 3000 ids spread over the sketch groups with
-    # values in [1, 1.05] (seven bf16 values, all within one sketch bin), the
-    # rest at -30.  The k-th id lies among ~3000 candidates, more than the
-    # fast kernel holds, so it hands every row over with its max and exp-sum;
-    # the value histogram counts the finite ids itself (the whole row is the
-    # nucleus) and takes the payload, ties in id order, from the top value.
+def test_ties_on_the_single_pass_kernel(A, orc):
+    # the same few-valued rows on aces_verify: whatever the kernel decides,
+    # ids of the crossing value are taken in id order
+    w = gen.make_workload(2, 2, 32000, "bf16", T=1.0, top_p=0.7, k=32, seed=42)
+    rng = np.random.default_rng(42)
+    vals = np.linspace(-2.0, 2.0, 40).astype(np.float32)
+    z = _bf16(vals[rng.integers(0, 40, size=(2, 3, 32000))])
+    counters, res = _run(A, orc, w, z)
+    assert res["checked_seqs"] >= 1
+
+
+def test_general_value_histogram_top_p_one_rows(A, orc):
+    # top_p = 1 on bf16 rows: 3000 ids with values in [1, 1.05] (seven bf16
+    # values), the rest at -30.  The value histogram counts the finite ids
+    # itself (the whole row is the nucleus) and takes the payload, ties in id
+    # order, from the top value.
     V, n_hot = 64000, 3000
     w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=1.0, k=64, seed=44)
     rng = np.random.default_rng(44)
@@ -170,24 +287,45 @@ def test_value_histogram_top_p_one_rows(A, orc):
     for b in range(2):
         for i in range(2):
             z[b, i, ids] = rng.uniform(1.0, 1.05, n_hot).astype(np.float32)
+    counters, res = _run(A, orc, w, _bf16(z), exact=True)
+    assert counters[FALLBACK] == 4 and counters[GEN_VALHIST] == 4 and counters[RADIX] == 0, counters
+    assert res["checked_seqs"] >= 1
+    # and on aces_verify
     counters, res = _run(A, orc, w, _bf16(z))
-    assert counters[0] == 4 and counters[6] == 4 and counters[4] == 0, counters
     assert res["checked_seqs"] >= 1
 
 
 def test_signed_zeros_on_the_general_path(A, orc):
     # -0 and +0 are one value (one order key): the nucleus and the payload take
     # them in id order whatever their signs.  Ten positive ids, then a run of
-    # 512 zeros of random sign (16 whole sketch groups, so the one-max-per-group
-    # bound cannot certify the row), the rest at -20.  Zero lies ~16000 bf16
-    # keys below a max near 1, beyond the value histogram's window, so the
-    # binned path takes the rows.
+    # 512 zeros of random sign, the rest at -20.  Zero lies ~16000 bf16 keys
+    # below a max near 1, beyond the value histogram's window, so the binned
+    # path takes the rows.
     V = 32000
     w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.999, k=64, seed=43)
     rng = np.random.default_rng(43)
     z = np.full((2, 2, V), -20.0, np.float32)
     z[:, :, 100:110] = rng.uniform(0.5, 1.0, size=(2, 2, 10)).astype(np.float32)
     z[:, :, 1024:1536] = np.where(rng.random((2, 2, 512)) < 0.5, np.float32(0.0), np.float32(-0.0))
+    counters, res = _run(A, orc, w, _bf16(z), exact=True)
+    assert counters[FALLBACK] == 4 and counters[GEN_VALHIST] == 0, counters
+    assert res["checked_seqs"] >= 1
+    # and on aces_verify (the list holds the zeros)
     counters, res = _run(A, orc, w, _bf16(z))
-    assert counters[0] == 4 and counters[6] == 0, counters
+    assert res["checked_seqs"] >= 1
+
+
+def test_general_radix_path(A, orc):
+    # float32 rows of 5000 tied ids at 0 (the rest at -30), top_p = 0.5: the
+    # crossing bin holds more ids than the binned path collects (2048), so
+    # the radix selection finishes the rows; ties go by id
+    V = 32768
+    w = gen.make_workload(2, 1, V, "f32", T=1.0, top_p=0.5, k=16, seed=49)
+    rng = np.random.default_rng(49)
+    z = np.full((2, 2, V), -30.0, np.float32)
+    for b in range(2):
+        for i in range(2):
+            z[b, i, rng.choice(V, 5000, replace=False)] = 0.0
+    counters, res = _run(A, orc, w, z, exact=True)
+    assert counters[FALLBACK] == 4 and counters[RADIX] >= 1, counters
     assert res["checked_seqs"] >= 1

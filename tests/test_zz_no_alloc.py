@@ -106,10 +106,10 @@ def test_same_inputs_twice_give_identical_outputs(lib):
 
 
 def test_largest_batch_runs_without_nucleus_lists(lib):
-    # B = 981 at K = 16 is the largest batch the scratch holds; its residual
+    # B = 923 at K = 16 is the largest batch the scratch holds; its residual
     # draws scan whole rows, aces_verify's use the stored nucleus lists.
     import paper_2609_02514_gb300 as A
-    w = gen.make_workload(981, 16, 1000, "f32", T=1.0, top_p=0.6, k=8, seed=44)
+    w = gen.make_workload(923, 16, 1000, "f32", T=1.0, top_p=0.6, k=8, seed=44)
     assert A.workspace_bytes(w.B, w.K, w.V, w.k) > SCRATCH_BYTES
     z, q, xt, u = _inputs(w)
     ref = A.verify(z, q, xt, u, w.T, w.top_p, w.k)
@@ -120,7 +120,7 @@ def test_largest_batch_runs_without_nucleus_lists(lib):
 
 
 def test_batch_beyond_the_scratch_is_rejected(lib):
-    B, K, V, k = 982, 16, 1000, 8          # needs more than ACES_NOALLOC_SCRATCH_BYTES
+    B, K, V, k = 924, 16, 1000, 8          # needs more than ACES_NOALLOC_SCRATCH_BYTES
     z = torch.zeros(B, K + 1, V, device="cuda")
     q = torch.full((B, K, V), 1.0 / V, device="cuda")
     xt = torch.zeros(B, K, dtype=torch.int32, device="cuda")
@@ -130,3 +130,19 @@ def test_batch_beyond_the_scratch_is_rejected(lib):
     assert _noalloc(lib, z, q, xt, u, w, k, o) == 2       # ACES_ERR_UNSUPPORTED
     torch.cuda.synchronize()
     assert (o["accept_len"] == -7).all()                   # nothing was launched
+
+
+def test_matches_the_oracle(lib, orc):
+    # one case compared with the float64 oracle directly (the other tests
+    # compare with aces_verify, itself compared with the oracle elsewhere)
+    from tests import parity
+    w = gen.make_workload(6, 8, 32000, "bf16", T=0.8, top_p=0.9, k=32, seed=45)
+    d = gen.generate(w)
+    z, q, xt, u = _inputs(w)
+    got = _outputs(w.B, w.K, w.k)
+    assert _noalloc(lib, z, q, xt, u, w, w.k, got) == 0
+    torch.cuda.synchronize()
+    g = {key: v.cpu().numpy() for key, v in got.items()}
+    o = orc.verify(d["z"], d["q"], d["xt"], d["u"], w.T, w.top_p, w.k)
+    res = parity.compare_verify(d, g, o, w.top_p, True, w.k)
+    assert res["checked_seqs"] >= w.B - 1, res
