@@ -43,7 +43,8 @@ VERIFY_KERNELS = ["k_rows_cap", "k_rows_general", "k_resolve_cut", "k_resolve_se
 # path counters at the start of the workspace (int32 words)
 PATHS = ["rows_on_general_kernel", "timeouts", "rows_value_histogram", "rows_bitonic_order",
          "general_rows_radix", "rows_cut_left_to_resolve", "general_rows_value_histogram",
-         "accept_tests_ranked_among_ties"]
+         "accept_tests_ranked_among_ties", "rows_published_depth", "rows_depth_from_finished_rows",
+         "rows_counted_twice"]
 
 
 # ---------------------------------------------------------------------------
@@ -371,7 +372,7 @@ def per_config(A, torch, dev, stream, peak, peak_kind, have=None, cpu=True):
             e1.record(stream)
         torch.cuda.synchronize()
         vms = statistics.median(e0.elapsed_time(e1) for e0, e1 in ev)
-        paths = dict(zip(PATHS, wsb[:32].view(torch.int32).cpu().numpy().tolist()))
+        paths = dict(zip(PATHS, wsb[:64].view(torch.int32).cpu().numpy().tolist()))
         paths.pop("timeouts")
         vb = verify_bytes(B, K, V, k, zsize, resid_q_count(out, K, k))
         for _ in range(3):
@@ -524,7 +525,7 @@ def main():
     al = out["accept_len"].cpu().numpy()
     n_rej = int((al < K).sum())
     n_resid_q = resid_q_count(out, K, k)
-    paths = dict(zip(PATHS, wsb[:32].view(torch.int32).cpu().numpy().tolist()))
+    paths = dict(zip(PATHS, wsb[:64].view(torch.int32).cpu().numpy().tolist()))
     paths.pop("timeouts")
     peak, peak_kind = measured_peak()
     vb = verify_bytes(B, K, V, k, zsize, n_resid_q)

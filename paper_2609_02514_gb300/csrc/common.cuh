@@ -354,21 +354,21 @@ struct SegSum {
 constexpr int NSEG_MAX = 16;
 constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual step
 
-constexpr int WS_COUNTERS = 256;  // bytes of path counters and depth hints at the start of the workspace
-constexpr int WS_DEPTH0 = 16;     // first of the 40 depth-histogram counters (int index)
+constexpr int WS_COUNTERS = 512;      // bytes of path counters and depth hints at the start of the workspace
+constexpr int WS_DEPTH = 16;          // first of the 40 depth counters of the row kernel's hints (int index)
 // Workspace layout (all offsets 16-byte aligned)
 struct Workspace {
-    int *fb_count;             // [64]  path counters and depth hints, cleared by every call: [0] rows handed to the
+    int *fb_count;             // [128] path counters and depth hints, cleared by every call: [0] rows handed to the
                                //       general kernel, [1] reserved (no kernel waits on another),
                                //       [2] rows captured by value histogram, [3] rows ordered by
                                //       bitonic sort, [4] rows the general kernel finished by radix
                                //       selection, [5] rows whose cut was left to the resolve step,
                                //       [6] rows the general kernel finished by value histogram,
                                //       [7] accept tests that ranked the draft token among ties,
-                               //       [8] rows that published the depth they needed,
-                               //       [16..55] how many rows needed each depth (the deeper of
-                               //       their crossing and payload end, in sample bins of T/4
-                               //       below the row's sample max)
+                               //       [8] rows that published the depths they needed,
+                               //       [16..55] how many rows had their crossing, [64..103] their
+                               //       payload end, at each depth (in sample bins of T/4 below
+                               //       the row's sample max)
     RowStat *stats;            // [rows]
     int *acc;                  // [B*K] accept bits
     int *fb_list;              // [rows]
@@ -460,7 +460,9 @@ struct RowArgs {
     int it_partial;        // iteration that reads the row's partial last tile (-1: none)
     float samp_frac;
     float inv_ws;          // sample bins per unit of logit: SPB / T
-    int nmin, npay;        // ids the capture must reach: for the nucleus and payload, for the payload list
+    int nmin;              // float32 first rows: ids the capture must reach
+    int sk_gpi, sk_ish;    // bfloat16 sketch: groups per thread and iteration (2: 4 chunks each; 1: 8
+                           // chunks of 2^sk_ish iterations)
     int force_fb;          // hand every row to the general kernel (the library's exact reference path)
 };
 

@@ -3,47 +3,45 @@
 // acceptance rule is the modified rejection sampling of Sec. II-A).
 //
 // One CTA of 256 threads per target row r = b*(K+1)+i, four CTAs per SM.
-// Every logit is read from HBM exactly once, with 16-byte loads, eight in
-// flight per thread.  The row is read in tiles of 32 chunks (one coalesced
-// 512-byte warp load) in the order t -> (t * pstride) mod ntile, so that the
-// first iteration (64 tiles) is a strided sample of the whole row.
+// Every logit is read from HBM once, with 16-byte loads, eight in flight per
+// thread.  The row is read in tiles of 32 chunks (one coalesced 512-byte warp
+// load) in the order t -> (t * pstride) mod ntile, so that the first
+// iteration (64 tiles) is a strided sample of the whole row.
 //
 //   stream    an online exp-sum in log2 units against an integer reference
 //             k_t = ceil(max z * log2(e)/T) (one paired FFMA per two logits,
-//             one ex2 per logit, exact power-of-two rescales) and the max.
-//   estimate  after the first iteration the sample's mass profile (bins of
-//             T/4 below its max) gives an estimate of the nucleus crossing
-//             and of the logit above which the payload lies; theta is put
-//             1.5 T below the estimated crossing (and low enough that about
-//             max(4k, 256) ids lie above it).  The estimate only decides what
-//             is kept: every result below is proved from exact sums.
-//   capture   every id >= theta is kept on chip while the row streams:
-//             list mode    (few ids expected; both dtypes): the id's 64-bit
-//                          order value goes to a shared-memory list;
-//             value mode   (bfloat16, many ids expected, theta > 0): one
-//                          shared-memory counter per bfloat16 value in a
-//                          window of 1024 values above theta is incremented,
-//                          and only ids above a second, higher threshold
-//                          (about max(4k, 64) ids) are listed.
+//             one ex2 per logit, exact power-of-two rescales), the max, and a
+//             running max shared by the CTA's warps.
+//   depth     D bounds how far below the row max the nucleus crossing (top_p
+//             = 1: the payload's end) lies: a quantile of the depths that the
+//             call's finished rows published, plus a margin (before any has
+//             finished: NSB bins of T/4).  D only decides what is kept; every
+//             result below is proved from exact sums.
+//   keep      bfloat16: every id >= (running max - D) increments a shared-
+//             memory counter of its bfloat16 value (a window of HW values),
+//             and a sketch keeps the max of every group of 4 to 8 chunks;
+//             float32: every 16-byte chunk holding an id >= the threshold is
+//             recorded (chunk and index).  The running max only rises, so at
+//             the end every id >= (row max - D) was kept.
 //   finish    from the exact row max and exp-sum, exact 2^-40 fixed-point
-//             masses prove that the nucleus crossing and the payload lie in
-//             the capture (else the row goes to the exact general kernel):
-//             list mode    the listed ids are binned by (m - z)/(T/8) with
-//                          exact masses; the bins up to the crossing bin are
-//                          ordered (direct ranking up to 512 ids, bitonic sort
-//                          above) and one warp finds the crossing;
-//             value mode   a prefix scan over the value counts gives the
-//                          crossing value, the number j of its ids inside the
-//                          nucleus and the payload's last value; the listed
-//                          payload ids are ranked.  When the crossing value's
-//                          ids are listed too, the j-th of them (in id order)
-//                          is the cut; otherwise the row keeps (value, j) and
-//                          the resolve step finds that id only for the rows it
-//                          draws from.
+//             masses give the nucleus crossing (else the row goes to the exact
+//             general kernel):
+//             bfloat16  one warp scans the value counts for the crossing
+//                       value, the number j of its ids inside the nucleus and
+//                       the payload's last value; the sketch's groups whose
+//                       max reaches that value are re-read and their ids at or
+//                       above it ordered.  When the crossing value's ids are
+//                       among them the j-th (in id order) is the cut;
+//                       otherwise the row keeps (value, j) and the resolve
+//                       step finds that id only for the rows it draws from.
+//             float32   the recorded ids are binned by (m - z)/(T/8) with
+//                       exact masses; the bins up to the crossing bin are
+//                       ordered (direct ranking up to 512 ids, bitonic sort
+//                       above) and one warp finds the crossing.
 //             Then the payload, the tail mass, the accept test of the draft
 //             token at this position and the per-row state; the CTA that
 //             finishes a sequence's last row draws its token when row pi's
-//             nucleus was listed.
+//             nucleus was kept.
 #include <climits>
 #include <mutex>
 #include <type_traits>
@@ -60,24 +58,31 @@ constexpr int NWC = NTC / 32;
 constexpr int UC = 8;               // 16-byte chunks per thread and iteration
 constexpr int TCH = 32;             // chunks per tile
 constexpr int TPI = NWC * UC;       // tiles per iteration
-constexpr int NSB = 40;             // sample bins (at most 64: two per lane of a warp)
-constexpr int SPB = 4;              // sample bins per temperature
-constexpr int MARGIN_BINS = 2;      // theta below the sample's crossing (0.5 T; the sample errs deep)
-constexpr int HW = 1024;            // value-mode window (bfloat16 values above theta)
+constexpr int NSB = 40;             // depth bins (of T/SPB) of the hints; D before any hint
+constexpr int SPB = 4;              // depth bins per temperature
+constexpr int MARGIN_BINS = 2;      // float32 first rows: theta below the sample's crossing
+constexpr int HINT_MIN = 32;        // finished rows before their depths set D
+constexpr int HINT_MARGIN = 2;      // depth bins of margin above that quantile
+constexpr float HINT_Q = 0.99f;     // the quantile of the finished rows' depths D covers
+// bfloat16
+constexpr int HW = 1024;            // counted values (bfloat16 bit patterns) per row
+constexpr int HEADROOM = 256;       // of them above the sample's max at least
+constexpr int SKG = 16384;          // sketch entries (group maxima, as 16-bit order keys)
+constexpr int PCAP = 1024;          // ids at or above the payload's last value
+constexpr int GCAP = 1024;          // sketch groups re-read
+constexpr int DEFER_IDS = 768;      // expected ids >= lim(max) below which they are counted after the stream
+constexpr int LIST_BF = SKG / 4;    // ids listed from the re-read groups (in the sketch's area)
+constexpr int SMEM_BF = HW * 4 + SKG * 2 + PCAP * 8;
+// float32
 constexpr int CREC = 1536;          // recorded chunks (16-byte chunk + its index) per row
 constexpr int LCAP = 2048;          // listed ids, expanded from the records after the stream
-constexpr int PCAP = 1024;          // value mode: payload candidates, crossing-value ids
-constexpr int VALUE_MIN = 6000;     // expected capture above which value mode is used
+constexpr int WCAP = 2048;          // work area: ordered candidates
+constexpr int SMEM_F32 = CREC * 20 + LCAP * 8 + NBIN * 4;
 constexpr int RANK_MAX = 512;       // ids ordered by direct ranking (more: bitonic sort)
-constexpr int WCAP = 2048;          // work area: ordered candidates, or payload + crossing-value ids
-// dynamic shared memory: [records: CREC x (16 + 4) bytes | list: LCAP u64 | window: HW u32];
-// the work area reuses the records once they are expanded
-constexpr int CAP_SMEM = CREC * 20 + LCAP * 8 + HW * 4;
-static_assert(WCAP * 8 <= CREC * 20, "the work area fits in the records' place");
-constexpr int HINT_MIN = 16;        // finished rows before their depths set theta
-constexpr int HINT_MARGIN = 1;      // sample bins of margin below that depth
-constexpr float HINT_Q = 0.99f;     // the quantile of the finished rows' depths theta covers
-static_assert(WS_DEPTH0 + NSB <= WS_COUNTERS / 4, "the depth histogram fits the counters area");
+static_assert(WS_DEPTH + NSB <= WS_COUNTERS / 4, "the depth histogram fits the counters area");
+static_assert(4 * NUC_CAP * 8 <= SMEM_BF && 4 * NUC_CAP * 8 <= SMEM_F32, "the draw's scratch fits");
+static_assert(GCAP * 4 <= HW * 4 && PCAP * 8 <= SKG * 2 && HW <= PCAP, "the aliased areas fit");
+static_assert(WCAP * 8 <= CREC * 20 && RANK_MAX * 2 <= LCAP, "the float32 work areas fit");
 
 __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     s = a + b;
@@ -202,6 +207,14 @@ __device__ __forceinline__ uint32_t chunk_hits(const uint4 &w, float th) {
     }
 }
 
+// adds 1 to the shared-memory counter at address addr when x < lim (one
+// predicated reduction: no branch)
+__device__ __forceinline__ void red_inc_lt(uint32_t addr, uint32_t x, uint32_t lim) {
+    asm volatile(
+        "{\n\t.reg .pred q;\n\tsetp.lt.u32 q, %1, %2;\n\t@q red.shared.add.u32 [%0], 1;\n\t}"
+        :: "r"(addr), "r"(x), "r"(lim) : "memory");
+}
+
 // bfloat16 order key of a bfloat16 bit pattern (keys sort like values, -0
 // and +0 share one key), and the value of a key
 __device__ __forceinline__ uint32_t key16(uint32_t b) {
@@ -283,28 +296,38 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     constexpr int EPC = E::EPC;
     constexpr bool BF = DT == ACES_BF16;
     extern __shared__ __align__(16) unsigned char smem[];
-    uint4 *rec_dat = reinterpret_cast<uint4 *>(smem);                                  // CREC
-    uint32_t *rec_idx = reinterpret_cast<uint32_t *>(smem + CREC * 16);                 // CREC
-    unsigned long long *list = reinterpret_cast<unsigned long long *>(smem + CREC * 20);  // LCAP
-    uint32_t *hist = reinterpret_cast<uint32_t *>(smem + CREC * 20 + LCAP * 8);         // HW (value mode)
-    unsigned long long *work = reinterpret_cast<unsigned long long *>(smem);            // WCAP, after expansion
-    // list-mode bin counts alias the value window (never both in one row)
-    uint32_t *bcnt = hist;
+    // bfloat16: [value counts: HW u32 | sketch: SKG u16 | ids >= the payload's
+    //           last value: PCAP u64]; the list of re-read groups reuses the
+    //           counts, the ordered ids the sketch, once each is read
+    uint32_t *hist = reinterpret_cast<uint32_t *>(smem);
+    uint16_t *sk = reinterpret_cast<uint16_t *>(smem + HW * 4);
+    unsigned long long *pay = reinterpret_cast<unsigned long long *>(smem + HW * 4 + SKG * 2);
+    uint32_t *glist = hist;
+    unsigned long long *sorted = reinterpret_cast<unsigned long long *>(sk);
+    // float32:  [records: CREC x (16 + 4) bytes | list: LCAP u64 | bin counts:
+    //           NBIN u32]; the work area reuses the records once they are expanded
+    uint4 *rec_dat = reinterpret_cast<uint4 *>(smem);
+    uint32_t *rec_idx = reinterpret_cast<uint32_t *>(smem + CREC * 16);
+    unsigned long long *list = reinterpret_cast<unsigned long long *>(smem + CREC * 20);
+    uint32_t *bcnt = reinterpret_cast<uint32_t *>(smem + CREC * 20 + LCAP * 8);
+    unsigned long long *work = reinterpret_cast<unsigned long long *>(smem);
 
-    __shared__ uint32_t sbin[NWC][NSB];  // per warp, relative to the warp's own max
+    __shared__ uint32_t sbin[NWC][NSB];  // float32 estimate: per warp, below the sample max
     __shared__ float redf[NWC], redk[NWC], redh[NWC], redl[NWC];
-    __shared__ int s_nrec, s_nl, s_mode, s_fb, s_n, s_bsel, s_nstar, s_L, s_npay, s_ntie, s_vs, s_vk, s_j, s_nn;
-    __shared__ float s_thlo, s_thpay, s_zx, s_m1;
-    __shared__ int s_xb;
+    __shared__ int s_nrec, s_nl, s_fb, s_n, s_bsel, s_nstar, s_L, s_npay, s_ng, s_nge, s_j, s_vs, s_vk, s_nnuc;
+    __shared__ float s_thlo, s_zx;
+    __shared__ int s_dbins, s_xb;  // s_dbins: D in depth bins (-1: no hints yet)
+    __shared__ uint32_t s_mr;  // order key of the running max
     __shared__ double s_S, s_Snuc;
     __shared__ float s_inv_S;
-    __shared__ unsigned long long s_cut, s_cumL_fx, s_above, s_cab;
+    __shared__ unsigned long long s_cut, s_cumL_fx;
     __shared__ unsigned long long s_redu[NWC];
 
     const int r = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const char *row = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
     const int nch = a.V / EPC, ntile = a.ntile;
+    const int nit = (ntile + TPI - 1) / TPI;
     const uint32_t NI = E::NEG_INF_WORD;
     const bool all_in = a.top_p >= 1.0f;
 
@@ -315,10 +338,24 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         iq = r % (a.K + 1);
         if (tid == 0 && iq < a.K) xb = a.xt[(size_t)bq * a.K + iq];
     }
-    for (int i = tid; i < NWC * NSB; i += NTC) (&sbin[0][0])[i] = 0u;
-    if (BF)
+    if (BF) {
         for (int i = tid; i < HW; i += NTC) hist[i] = 0u;
-    if (tid == 0) s_nrec = 0;
+    } else {
+        for (int i = tid; i < NWC * NSB; i += NTC) (&sbin[0][0])[i] = 0u;
+    }
+    if (tid == 0) {
+        s_nrec = 0;
+        s_nl = 0;
+        s_mr = fkey(-INFINITY);
+    }
+    // the depths published by the call's finished rows (read by warp 0 only,
+    // once: they change while this row streams)
+    int hr = 0, hc0 = 0, hc1 = 0;
+    if (wid == 0) {
+        hr = __ldcg(&a.ws.fb_count[8]);
+        hc0 = 2 * lane < NSB ? __ldcg(&a.ws.fb_count[WS_DEPTH + 2 * lane]) : 0;
+        hc1 = 2 * lane + 1 < NSB ? __ldcg(&a.ws.fb_count[WS_DEPTH + 2 * lane + 1]) : 0;
+    }
 
     // ---- stream ----
     float k_t = -1e30f, m_t = -INFINITY, s_t = 0.f, e_t = 0.f;
@@ -346,16 +383,20 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         for (int u = 0; u < UC; ++u) hb |= (uint32_t)(max2_value<DT>(chunk_max2<DT>(w[u])) >= th) << u;
         return hb;
     };
-    // max and exp-sum of this iteration; returns mask_of(th)
-    auto math = [&](float th) -> uint32_t {
-        float im = -INFINITY;
+    // max and exp-sum of this iteration; returns mask_of(th), the iteration's
+    // max in im and the maxima of chunks 0..3 and 4..7 in g0, g1
+    auto math = [&](float th, float &im, float &g0, float &g1) -> uint32_t {
         uint32_t hb = 0u;
+        g0 = -INFINITY;
+        g1 = -INFINITY;
 #pragma unroll
         for (int u = 0; u < UC; ++u) {
             const float cmx = max2_value<DT>(chunk_max2<DT>(w[u]));
-            im = fmaxf(im, cmx);
+            if (u < UC / 2) g0 = fmaxf(g0, cmx);
+            else g1 = fmaxf(g1, cmx);
             hb |= (uint32_t)(cmx >= th) << u;
         }
+        im = fmaxf(g0, g1);
         m_t = fmaxf(m_t, im);
         const float gk = im * a.c;
         if (gk > k_t) {
@@ -372,272 +413,781 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         s_t = t;
         return hb;
     };
-    // records the chunks in hb (those holding an id >= the capture
-    // threshold): one vote per iteration, one warp-aggregated atomic per chunk
-    // position that has any; the ids are extracted after the stream
-    auto record_hits = [&](uint32_t hb) {
-        if (!__any_sync(0xffffffffu, hb != 0u)) return;
-        int tile = tile0;
+    // the running max of the CTA (a lower bound of the row max at any time)
+    auto publish_max = [&](float im) {
+        const float wm = warp_max(im);
+        if (lane == 0 && wm > -INFINITY) atomicMax(&s_mr, fkey(wm));
+    };
+    auto running_max = [&]() -> float { return fkey_inv(*reinterpret_cast<volatile uint32_t *>(&s_mr)); };
+
+    // iteration 0: a strided sample (1/8 to 1/16 of a large row, spread over it)
+    float im, g0, g1;
+    load(0);
+    math(INFINITY, im, g0, g1);
+    // D: how far below the row max the nucleus crossing (top_p = 1: the
+    // payload's end) can lie.  Rows of this call that have finished published
+    // their depths (in bins of T/4 below their max); the HINT_Q quantile of
+    // those depths, plus a margin, sets D (in bins; -1: before HINT_MIN rows
+    // have finished, a fixed NSB bins).  One value for the whole CTA.
+    if (wid == 0) {
+        int inc = hc0 + hc1;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= o) inc += t;
+        }
+        const float need = HINT_Q * (float)__shfl_sync(0xffffffffu, inc, 31);
+        const int hb = (float)(inc - hc1) >= need ? 2 * lane : ((float)inc >= need ? 2 * lane + 1 : NSB);
+        const unsigned bal = __ballot_sync(0xffffffffu, hb < NSB);
+        const int hq = bal ? __shfl_sync(0xffffffffu, hb, __ffs(bal) - 1) : NSB - 1;
+        if (lane == 0) s_dbins = hr >= HINT_MIN ? min(hq + HINT_MARGIN, NSB - 1) + 1 : -1;
+    }
+    publish_max(im);
+    __syncthreads();
+    const float m1 = running_max();  // the sample's max
+    const bool have = m1 > -INFINITY && m1 < INFINITY;
+    const int hbins = s_dbins;
+    const bool hinted = have && hbins > 0;
+    const float D = (float)(hinted ? hbins : NSB) * (a.T / SPB);
+
+    // dependent loads of the accept test, consumed at the end
+    float zx = 0.f, qx = 0.f, ux = 0.f;
+    int L = 0;
+    unsigned long long *ord = nullptr;  // the payload in order (and, when kept, the nucleus)
+    int lazy = 0;
+    int nnuc = -1;  // nucleus ids written to the row's list (-1: none)
+    float m = -INFINITY, kref = -1e30f;
+    double S = 0.0;
+    float v_need = 0.0f;  // the crossing (top_p = 1: the payload's end), for the hints
+
+    // reduces the row max, the reference and the exp-sum (fp32 two-sum tree,
+    // fp64 in warp 0); true when the row is not a distribution (handled)
+    auto finish_sums = [&]() -> bool {
+        if (xb >= 0 && xb < a.V) {
+            zx = E::load1(row, xb);
+            qx = __ldg(a.q + ((size_t)bq * a.K + iq) * a.V + xb);
+            ux = __ldg(a.u + (size_t)bq * (a.K + 1) + iq);
+        }
+        {
+            const float mw = warp_max(m_t), kw = warp_max(k_t);
+            if (lane == 0) {
+                redf[wid] = mw;
+                redk[wid] = kw;
+            }
+        }
+        __syncthreads();
+        m = redf[0];
+        kref = redk[0];
 #pragma unroll
-        for (int u = 0; u < UC; ++u) {
-            const bool hit = (hb >> u) & 1u;
-            const unsigned bal = __ballot_sync(0xffffffffu, hit);
-            if (bal != 0u) {
-                const int lead = __ffs(bal) - 1;
-                int base = 0;
-                if (lane == lead) base = atomicAdd(&s_nrec, __popc(bal));
-                base = __shfl_sync(0xffffffffu, base, lead);
-                if (hit) {
-                    const int at = base + __popc(bal & ((1u << lane) - 1u));
-                    if (at < CREC && ACES_IN(at, CREC)) {
-                        rec_dat[at] = w[u];
-                        rec_idx[at] = (uint32_t)(tile * TCH + lane);
+        for (int i = 1; i < NWC; ++i) {
+            m = fmaxf(m, redf[i]);
+            kref = fmaxf(kref, redk[i]);
+        }
+        {
+            const float f = pow2_int(fmaxf(k_t - kref, -1000.0f));
+            float hi = s_t * f, lo = e_t * f;
+            for (int o = 16; o > 0; o >>= 1) {
+                const float h2 = __shfl_xor_sync(0xffffffffu, hi, o);
+                const float l2 = __shfl_xor_sync(0xffffffffu, lo, o);
+                float sm, er;
+                two_sum(hi, h2, sm, er);
+                lo = lo + l2 + er;
+                hi = sm;
+            }
+            if (lane == 0) {
+                redh[wid] = hi;
+                redl[wid] = lo;
+            }
+        }
+        __syncthreads();
+        if (wid == 0) {
+            const double Sw = warp0_mass(redh, redl, lane);
+            if (lane == 0) {
+                s_S = Sw;
+                s_fb = 0;
+                s_nstar = INT_MAX;
+            }
+        }
+        __syncthreads();
+        S = s_S;
+        if (!(S > 0.0 && S < 1e300) || !(m < INFINITY) || !(kref < 1e30f)) {
+            nonfinite_row<NTC>(a, r);
+            row_finished(a, r, smem);
+            return true;
+        }
+        return false;
+    };
+
+    if constexpr (BF) {
+        // ================= bfloat16: value counts and sketch =================
+        // Every id >= lim(running max) is counted in the window of HW values
+        // [thb0, thb0 + HW) (positive bit patterns, which sort like the
+        // values); the running max only rises, so at the end every id >=
+        // lim(row max) has been counted.  The sketch keeps the max of every
+        // group of chunks (4 or 8 chunks of one thread and iteration, or 8
+        // chunks of 2^ish iterations).
+        uint32_t thb0 = 1u;
+        bool count_on = false;
+        if (have && m1 > 0.0f) {
+            const float t = m1 - D;
+            int lo = t > 0.0f ? (int)__bfloat16_as_ushort(__float2bfloat16_rd(t)) : 1;
+            lo = max(lo, (int)(__float_as_uint(m1) >> 16) + HEADROOM - (HW - 1));
+            lo = max(lo, 1);
+            if (lo + HW - 1 <= 0x7F7F) {  // (then negative values, inf and NaN fall outside)
+                count_on = true;
+                thb0 = (uint32_t)lo;
+            }
+        }
+        auto lim_of = [&](float mr) -> uint32_t {
+            const float t = mr - D;
+            uint32_t b = t > 0.0f ? (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rd(t)) : 0u;
+            b = b > thb0 ? b : thb0;
+            return b < thb0 + HW ? b : thb0 + HW;
+        };
+        // (the counts' shared-memory address, offset so that a value's bit
+        // pattern times 4 indexes its counter)
+        const uint32_t hbase = (uint32_t)__cvta_generic_to_shared(hist) - thb0 * 4u;
+        auto count_hits = [&](uint32_t hb, uint32_t thb) {
+            if (hb == 0u) return;  // (no chunk of this thread reaches thb)
+            const uint32_t span = thb0 + HW - thb;
+#pragma unroll
+            for (int u = 0; u < UC; ++u) {
+                if ((hb >> u) & 1u) {
+                    const uint32_t wd[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint32_t lo = wd[q] & 0xFFFFu, hi = wd[q] >> 16;
+#ifdef ACES_CHECKED
+                        if (lo - thb < span && ACES_IN(lo - thb0, HW)) atomicAdd(&hist[lo - thb0], 1u);
+                        if (hi - thb < span && ACES_IN(hi - thb0, HW)) atomicAdd(&hist[hi - thb0], 1u);
+#else
+                        red_inc_lt(hbase + lo * 4u, lo - thb, span);
+                        red_inc_lt(hbase + hi * 4u, hi - thb, span);
+#endif
                     }
                 }
             }
-            tile += a.pstride_w;
-            if (tile >= ntile) tile -= ntile;
-        }
-    };
-    // value mode: one count per id of each bfloat16 value in [theta, theta + HW
-    // values), branch-free (theta > 0: the bit patterns of positive values are
-    // their order, and every other id falls outside the window); ids above the
-    // window are caught by the max check at the end
-    auto count_all = [&](uint32_t thb) {
-#pragma unroll
-        for (int u = 0; u < UC; ++u) {
-            const uint32_t wd[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint32_t rl = (wd[q] & 0xFFFFu) - thb, rh = (wd[q] >> 16) - thb;
-                if (rl < (uint32_t)HW && ACES_IN(rl, HW)) atomicAdd(&hist[rl], 1u);
-                if (rh < (uint32_t)HW && ACES_IN(rh, HW)) atomicAdd(&hist[rh], 1u);
-            }
-        }
-    };
-
-    // iteration 0: the sample.  Each warp bins its ids near its own max
-    // (bins of T/SPB, NSB of them); warp 0 aligns the warps' bins and takes
-    // the sample's mass from the exact exp-sums.
-    load(0);
-    math(INFINITY);
-    {
-        const float mw = warp_max(m_t);
-        // every id of the sample within NSB bins of the warp's max is binned
-        // (few are); chunks holding none are skipped by a vote
-        if (mw > -INFINITY && mw < INFINITY) {
-#pragma unroll
-            for (int u = 0; u < UC; ++u) {
-                const float cmx = max2_value<DT>(chunk_max2<DT>(w[u]));
-                if (!__any_sync(0xffffffffu, (mw - cmx) * a.inv_ws < (float)NSB)) continue;
-#pragma unroll 1  // (unrolled, the independent atomics spill registers)
-                for (int e = 0; e < EPC; ++e) {
-                    const float d = (mw - chunk_elem<DT>(w[u], e)) * a.inv_ws;
-                    if (d < (float)NSB && ACES_IN((int)d, NSB)) atomicAdd(&sbin[wid][(int)d], 1u);
+        };
+        const int gpi = a.sk_gpi, ish = a.sk_ish;
+        uint32_t gacc = 0u;
+        auto sketch_put = [&](int it) {
+            const uint32_t k0 = key16(__float_as_uint(g0) >> 16), k1 = key16(__float_as_uint(g1) >> 16);
+            if (gpi == 2) {
+                const int s2 = it * NTC + tid;
+                if (ACES_IN(2 * s2 + 1, SKG)) reinterpret_cast<uint32_t *>(sk)[s2] = k0 | (k1 << 16);
+            } else {
+                gacc = max(gacc, max(k0, k1));
+                if (((it + 1) & ((1 << ish) - 1)) == 0 || it == nit - 1) {
+                    const int s1 = (it >> ish) * NTC + tid;
+                    if (ACES_IN(s1, SKG)) sk[s1] = (uint16_t)gacc;
+                    gacc = 0u;
                 }
             }
-        }
-        // the sample's mass: this warp's exp-sum against its largest reference
-        const float kw = warp_max(k_t);
-        float sw = (s_t + e_t) * pow2_int(fmaxf(k_t - kw, -1000.0f));
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) sw += __shfl_xor_sync(0xffffffffu, sw, o);
-        if (lane == 0) {
-            redf[wid] = mw;
-            redk[wid] = kw;
-            redh[wid] = sw;
-        }
-    }
-    __syncthreads();
-    float m1 = redf[0];
-#pragma unroll
-    for (int i = 1; i < NWC; ++i) m1 = fmaxf(m1, redf[i]);
-    const bool have = m1 > -INFINITY && m1 < INFINITY;
-    if (wid == 0 && have) {
-        // bins 2 * lane and 2 * lane + 1 below m1, from the warps' bins shifted
-        // by the (rounded) distance of their maxima; the sample's mass in units
-        // of 2^((z - m1) c) from the warps' sums
-        uint32_t c0 = 0u, c1 = 0u;
-        float M = 0.0f;
-#pragma unroll
-        for (int i = 0; i < NWC; ++i) {
-            const float mwi = redf[i];
-            if (!(mwi > -INFINITY)) continue;
-            const int off = __float2int_rn((m1 - mwi) * a.inv_ws);
-            const int s0 = 2 * lane - off, s1 = 2 * lane + 1 - off;
-            if (s0 >= 0 && s0 < NSB) c0 += sbin[i][s0];
-            if (s1 >= 0 && s1 < NSB) c1 += sbin[i][s1];
-            M += redh[i] * ex2(redk[i] - m1 * a.c);
-        }
-        constexpr float L2B = 1.4426950408889634f / SPB;
-        const float ms0 = (float)c0 * ex2(-(2 * lane + 0.5f) * L2B), ms1 = (float)c1 * ex2(-(2 * lane + 1.5f) * L2B);
-        float pm = ms0 + ms1;
-        uint32_t pc = c0 + c1;
-        for (int o = 1; o < 32; o <<= 1) {
-            const float tm = __shfl_up_sync(0xffffffffu, pm, o);
-            const uint32_t tc = __shfl_up_sync(0xffffffffu, pc, o);
-            if (lane >= o) {
-                pm += tm;
-                pc += tc;
-            }
-        }
-        const float pm0 = pm - ms1, pc0f = (float)(pc - c1);  // cumulative through bin 2*lane
-        // first bin whose cumulative reaches a target (NSB when none)
-        auto first_bin = [&](bool h0, bool h1) -> int {
-            const int hb = h0 ? 2 * lane : (h1 ? 2 * lane + 1 : NSB);
-            const unsigned bal = __ballot_sync(0xffffffffu, hb < NSB);
-            return bal ? __shfl_sync(0xffffffffu, hb, __ffs(bal) - 1) : NSB;
         };
-        const float f = a.samp_frac;
-        auto bin_of_count = [&](float n) { return first_bin(pc0f >= n * f, (float)pc >= n * f); };
-        int blo;
-        if (all_in) {
-            blo = bin_of_count((float)a.nmin);
-        } else {
-            const float tm = a.top_p * M;
-            const int bx = first_bin(pm0 >= tm, pm >= tm);
-            blo = max(bx + MARGIN_BINS, bin_of_count((float)a.nmin));
-        }
-        // rows of this call already finished: the depth (crossing or payload
-        // end, whichever is deeper) that HINT_Q of them needed sets theta
-        // instead; a row that needs more falls back to the exact kernel
-        const int hrows = __ldcg(&a.ws.fb_count[8]);
-        if (hrows >= HINT_MIN) {
-            const int h0 = 2 * lane < NSB ? __ldcg(&a.ws.fb_count[WS_DEPTH0 + 2 * lane]) : 0;
-            const int h1 = 2 * lane + 1 < NSB ? __ldcg(&a.ws.fb_count[WS_DEPTH0 + 2 * lane + 1]) : 0;
-            int hc = h0 + h1, hi = hc;
-            for (int o = 1; o < 32; o <<= 1) {
-                const int t = __shfl_up_sync(0xffffffffu, hi, o);
-                if (lane >= o) hi += t;
-            }
-            const int htot = __shfl_sync(0xffffffffu, hi, 31);
-            const float need = HINT_Q * (float)htot;
-            const int hb0 = (float)(hi - h1) >= need ? 2 * lane : ((float)hi >= need ? 2 * lane + 1 : NSB);
-            const unsigned hbal = __ballot_sync(0xffffffffu, hb0 < NSB);
-            const int hd = hbal ? __shfl_sync(0xffffffffu, hb0, __ffs(hbal) - 1) : NSB - 1;
-            blo = hd + HINT_MARGIN;
-            (void)hc;
-        }
-        blo = min(blo, NSB - 1);
-        // expected ids >= theta
-        const float cum_lo = __shfl_sync(0xffffffffu, (blo & 1) ? (float)pc : pc0f, blo >> 1);
-        const float n_est = cum_lo / f;
-        const float thlo = m1 - (float)(blo + 1) * (a.T / SPB);
-        int mode = 0;  // list mode
-        float thpay = thlo;
-        if (BF && !all_in && n_est > (float)VALUE_MIN && thlo > 0.0f) {
-            mode = 1;  // value mode
-            const int bp = min(bin_of_count((float)a.npay), blo);
-            thpay = m1 - (float)(bp + 1) * (a.T / SPB);
-        }
-        if (lane == 0) {
-            float tl = thlo, tp = thpay;
-            if (BF) {  // thresholds are bfloat16 values (rounded down)
-                tl = __bfloat162float(__float2bfloat16_rd(tl));
-                tp = __bfloat162float(__float2bfloat16_rd(tp));
-                if (mode == 1 && !(tl > 0.0f)) tl = __uint_as_float(0x00010000u);  // smallest positive
-                if (tp < tl) tp = tl;
-            }
-            s_thlo = tl;
-            s_thpay = tp;
-            s_mode = mode;
-            s_m1 = m1;
-        }
-    }
-    __syncthreads();
-    const int mode = have ? s_mode : 0;
-    const float thlo = have ? s_thlo : INFINITY;  // no estimate: keep nothing
-    const float thpay = have ? s_thpay : INFINITY;
-    const int nit = (ntile + TPI - 1) / TPI;
-    if (mode == 0) {
-        uint32_t hb = mask_of(thlo);  // (iteration 0 is loaded and summed)
-        for (int it = 0; it < nit; ++it) {
-            if (it > 0) {
-                tile0 += a.pstride_it;
-                if (tile0 >= ntile) tile0 -= ntile;
-                load(it);
-                hb = math(thlo);
-            }
-            record_hits(hb);
-        }
-    } else {
-        const uint32_t thb = __float_as_uint(thlo) >> 16;  // bit pattern of theta (> 0)
-        uint32_t hb = mask_of(thpay);
-        for (int it = 0; it < nit; ++it) {
-            if (it > 0) {
-                tile0 += a.pstride_it;
-                if (tile0 >= ntile) tile0 -= ntile;
-                load(it);
-                hb = math(thpay);
-            }
-            count_all(thb);
-            record_hits(hb);
-        }
-    }
-    // dependent loads of the accept test, consumed at the end
-    float zx = 0.f, qx = 0.f, ux = 0.f;
-    if (xb >= 0 && xb < a.V) {
-        zx = E::load1(row, xb);
-        qx = __ldg(a.q + ((size_t)bq * a.K + iq) * a.V + xb);
-        ux = __ldg(a.u + (size_t)bq * (a.K + 1) + iq);
-    }
-
-    // ---- row max, reference and exp-sum (fp32 two-sum tree, fp64 in warp 0) ----
-    {
-        const float mw = warp_max(m_t), kw = warp_max(k_t);
-        if (lane == 0) {
-            redf[wid] = mw;
-            redk[wid] = kw;
-        }
-    }
-    __syncthreads();
-    float m = redf[0], kref = redk[0];
+        // Rows expected to hold few ids >= lim(m1) (the sample's count,
+        // scaled) defer the counting: the stream only sums and keeps the
+        // sketch, and after it the groups that reach the row's own lim(m)
+        // are read back, their ids listed and counted.  Others count while
+        // streaming.
+        int defer = 0;
+        if (count_on) {
+            const float thf0 = __uint_as_float(lim_of(m1) << 16);
+            uint32_t cnt = 0u;
 #pragma unroll
-    for (int i = 1; i < NWC; ++i) {
-        m = fmaxf(m, redf[i]);
-        kref = fmaxf(kref, redk[i]);
-    }
-    {
-        const float f = pow2_int(fmaxf(k_t - kref, -1000.0f));
-        float hi = s_t * f, lo = e_t * f;
-        for (int o = 16; o > 0; o >>= 1) {
-            const float h2 = __shfl_xor_sync(0xffffffffu, hi, o);
-            const float l2 = __shfl_xor_sync(0xffffffffu, lo, o);
-            float sm, er;
-            two_sum(hi, h2, sm, er);
-            lo = lo + l2 + er;
-            hi = sm;
+            for (int u = 0; u < UC; ++u) cnt += __popc(chunk_hits<DT>(w[u], thf0));
+            cnt = __reduce_add_sync(0xffffffffu, cnt);
+            if (lane == 0) atomicAdd(&s_nl, (int)cnt);
+            __syncthreads();
+            defer = (float)s_nl < (float)DEFER_IDS * a.samp_frac;
         }
-        if (lane == 0) {
-            redh[wid] = hi;
-            redl[wid] = lo;
+        if (defer) {
+            for (int it = 0; it < nit; ++it) {
+                if (it > 0) {
+                    tile0 += a.pstride_it;
+                    if (tile0 >= ntile) tile0 -= ntile;
+                    load(it);
+                    math(INFINITY, im, g0, g1);
+                }
+                sketch_put(it);
+            }
+        } else {
+            uint32_t thb = count_on ? lim_of(m1) : 0u;
+            float thf = count_on ? __uint_as_float(thb << 16) : INFINITY;
+            uint32_t hb = mask_of(thf);  // (iteration 0 is loaded and summed)
+            for (int it = 0; it < nit; ++it) {
+                if (it > 0) {
+                    tile0 += a.pstride_it;
+                    if (tile0 >= ntile) tile0 -= ntile;
+                    load(it);
+                    if (count_on) {
+                        thb = lim_of(running_max());
+                        thf = __uint_as_float(thb << 16);
+                    }
+                    hb = math(thf, im, g0, g1);
+                    publish_max(im);
+                }
+                if (count_on) count_hits(hb, thb);
+                sketch_put(it);
+            }
         }
-    }
-    __syncthreads();
-    if (wid == 0) {
-        const double S = warp0_mass(redh, redl, lane);
-        if (lane == 0) {
-            s_S = S;
-            s_fb = 0;
-            s_nstar = INT_MAX;
+        if (finish_sums()) return;
+        const uint32_t km = __float_as_uint(m) >> 16;
+        if (a.force_fb || !(m > 0.0f)) {
+            if (tid == 0) fallback_row(a, r, m, kref, S);
+            return;
         }
-    }
-    __syncthreads();
-    const double S = s_S;
-    if (!(S > 0.0 && S < 1e300) || !(m < INFINITY) || !(kref < 1e30f)) {
-        nonfinite_row<NTC>(a, r);
-        row_finished(a, r, smem);
-        return;
-    }
-    const int nrec = s_nrec;
-    if (a.force_fb || nrec > CREC) {
-        if (tid == 0) fallback_row(a, r, m, kref, S);
-        return;
-    }
-    // expand the records: the ids >= the capture threshold of every recorded
-    // chunk (all such ids lie in recorded chunks), as 64-bit order values
-    {
-        const float th = mode == 0 ? thlo : thpay;
+        const unsigned long long tg = all_in ? 0ull : (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
+        auto vmass = [&](int idx) { return id_fx(val16(0x8000u + thb0 + (uint32_t)idx), a.c, kref); };
+        unsigned long long *emass = pay;  // (until the re-read) the mass of one id of each counted value
+        // ---- the crossing, the payload's end and the values to re-read,
+        // from the counts of values thc..m (warp 0).  Returns 0, or 1 when
+        // they lie below the counted values, 2 when more ids than the
+        // re-read keeps share the payload's last value ----
+        auto scan = [&](uint32_t thc) -> int {
+            if (wid == 0) {
+                const int top = (int)(km - thb0), lo = (int)(thc - thb0);
+                const int per = (top - lo + 32) >> 5;
+                const int b0 = top - lane * per;  // this lane's values: b0, b0 - 1, ... (>= lo)
+                unsigned long long lm = 0ull, lc = 0ull;
+                for (int i = 0; i < per; ++i) {
+                    const int idx = b0 - i;
+                    if (idx < lo) break;
+                    const uint32_t cn = hist[idx];
+                    if (cn) {
+                        const unsigned long long e1 = vmass(idx);
+                        if (ACES_IN(idx, PCAP)) emass[idx] = e1;
+                        lm += (unsigned long long)cn * e1;
+                        lc += cn;
+                    }
+                }
+                unsigned long long incm = lm, incc = lc;
+                for (int o = 1; o < 32; o <<= 1) {
+                    const unsigned long long tm = __shfl_up_sync(0xffffffffu, incm, o);
+                    const unsigned long long tc = __shfl_up_sync(0xffffffffu, incc, o);
+                    if (lane >= o) {
+                        incm += tm;
+                        incc += tc;
+                    }
+                }
+                const unsigned long long exm = incm - lm, exc = incc - lc;
+                const unsigned long long totc = __shfl_sync(0xffffffffu, incc, 31);
+                int fail = 0, vs = -1, jj = 0;
+                unsigned long long above = 0ull, cab = 0ull, cnvs = 0ull;
+                if (!all_in) {
+                    if (exm < tg && incm >= tg) {
+                        unsigned long long cm = exm, cc = exc;
+                        for (int i = 0; i < per; ++i) {
+                            const int idx = b0 - i;
+                            if (idx < lo) break;
+                            const uint32_t cn = hist[idx];
+                            if (!cn) continue;
+                            const unsigned long long e1 = emass[idx];
+                            const unsigned long long mm = (unsigned long long)cn * e1;
+                            if (cm + mm >= tg) {
+                                vs = idx;
+                                above = cm;
+                                cab = cc;
+                                cnvs = cn;
+                                // the fewest ids of this value reaching the target
+                                const unsigned long long rem = tg - cm;
+                                unsigned long long q = (unsigned long long)((double)rem / (double)e1);
+                                while (q * e1 < rem) ++q;
+                                while (q > 1ull && (q - 1ull) * e1 >= rem) --q;
+                                jj = (int)q;
+                                break;
+                            }
+                            cm += mm;
+                            cc += cn;
+                        }
+                    }
+                    const unsigned bal = __ballot_sync(0xffffffffu, vs >= 0);
+                    if (bal) {
+                        const int src = __ffs(bal) - 1;
+                        vs = __shfl_sync(0xffffffffu, vs, src);
+                        jj = __shfl_sync(0xffffffffu, jj, src);
+                        above = __shfl_sync(0xffffffffu, above, src);
+                        cab = __shfl_sync(0xffffffffu, cab, src);
+                        cnvs = __shfl_sync(0xffffffffu, cnvs, src);
+                    } else {
+                        fail = 1;
+                    }
+                }
+                const unsigned long long nn = all_in ? (unsigned long long)a.V : cab + (unsigned long long)jj;
+                const int Lw = fail ? 0 : (int)(nn < (unsigned long long)a.k ? nn : (unsigned long long)a.k);
+                if (!fail && (unsigned long long)Lw > totc) fail = 1;  // (top_p = 1) the payload reaches below them
+                int vk = -1;
+                unsigned long long cabk = 0ull, mabk = 0ull, cnk = 0ull;
+                if (!fail && Lw > 0) {
+                    const unsigned long long Lu = (unsigned long long)Lw;
+                    if (exc < Lu && incc >= Lu) {
+                        unsigned long long cm = exm, cc = exc;
+                        for (int i = 0; i < per; ++i) {
+                            const int idx = b0 - i;
+                            if (idx < lo) break;
+                            const uint32_t cn = hist[idx];
+                            if (!cn) continue;
+                            if (cc + cn >= Lu) {
+                                vk = idx;
+                                cabk = cc;
+                                mabk = cm;
+                                cnk = cn;
+                                break;
+                            }
+                            cc += cn;
+                            cm += (unsigned long long)cn * emass[idx];
+                        }
+                    }
+                    const unsigned bal = __ballot_sync(0xffffffffu, vk >= 0);
+                    const int src = bal ? __ffs(bal) - 1 : 0;
+                    vk = __shfl_sync(0xffffffffu, vk, src);
+                    cabk = __shfl_sync(0xffffffffu, cabk, src);
+                    mabk = __shfl_sync(0xffffffffu, mabk, src);
+                    cnk = __shfl_sync(0xffffffffu, cnk, src);
+                    if (vk < 0) fail = 1;
+                }
+                // the values to re-read: down to the crossing value when the
+                // nucleus is short (then it is kept and the cut is exact),
+                // else down to the payload's last value
+                int vr = -1;
+                unsigned long long nge = 0ull;
+                if (!fail) {
+                    if (!all_in && cab + cnvs <= (unsigned long long)PCAP && nn <= (unsigned long long)NUC_CAP) {
+                        vr = vs;
+                        nge = cab + cnvs;
+                    } else if (Lw > 0) {
+                        vr = vk;
+                        nge = cabk + cnk;
+                        if (nge > (unsigned long long)PCAP) fail = 2;
+                    }
+                }
+                if (lane == 0) {
+                    s_fb = fail;
+                    s_vs = vs;
+                    s_vk = vr;
+                    s_j = jj;
+                    s_L = Lw;
+                    s_nnuc = all_in ? -1 : (int)(nn < (unsigned long long)INT_MAX ? nn : (unsigned long long)INT_MAX);
+                    s_nge = (int)nge;
+                    s_ng = 0;
+                    s_npay = 0;
+                    if (!fail) {
+                        const unsigned long long ek = vk >= 0 ? emass[vk] : 0ull;
+                        s_cumL_fx = mabk + ((unsigned long long)Lw - cabk) * ek;
+                        s_Snuc = all_in ? S : (double)(above + (unsigned long long)jj * emass[vs]) * FX_INV;
+                        s_inv_S = inv_mass(s_Snuc);
+                    }
+                }
+            }
+            __syncthreads();
+            return s_fb;
+        };
+        // ---- reading groups of the sketch back ----
+        const int ng_all = gpi == 2 ? nit * NTC * 2 : ((nit + (1 << ish) - 1) >> ish) * NTC;
+        // cnt items of each lane get consecutive places from *ctr (one atomic
+        // per warp); returns the lane's first place (all lanes of the warp)
+        auto warp_place = [&](int cnt, int *ctr) -> int {
+            int inc = cnt;
+            for (int o = 1; o < 32; o <<= 1) {
+                const int t = __shfl_up_sync(0xffffffffu, inc, o);
+                if (lane >= o) inc += t;
+            }
+            int base = 0;
+            if (lane == 31 && inc > 0) base = atomicAdd(ctr, inc);
+            return __shfl_sync(0xffffffffu, base, 31) + inc - cnt;
+        };
+        // lists in gl the slots whose group max (16-bit order key) reaches
+        // key; returns their count (all threads)
+        auto compact = [&](uint32_t key, uint32_t *gl) -> int {
+            if (tid == 0) s_ng = 0;
+            __syncthreads();
+            const int per_t = ng_all / NTC;  // (at most 64: slot i * NTC + tid)
+            unsigned long long hm = 0ull;
+            for (int i = 0; i < per_t; ++i) {
+                const int slot = i * NTC + tid;
+                if (ACES_IN(slot, SKG) && sk[slot] >= key) hm |= 1ull << i;
+            }
+            int at = warp_place(__popcll(hm), &s_ng);
+            while (hm) {
+                const int i = __ffsll((long long)hm) - 1;
+                hm &= hm - 1ull;
+                if (at < GCAP && ACES_IN(at, GCAP)) gl[at] = (uint32_t)(i * NTC + tid);
+                ++at;
+            }
+            __syncthreads();
+            return s_ng;
+        };
+        // reads the ng groups of gl (one per thread, four chunks at a time) and
+        // hands every id whose bit pattern is >= vb (> 0) to put(place, bits,
+        // id), places counted by *ctr
+        auto reread = [&](const uint32_t *gl, int ng, uint32_t vb, int *ctr, auto put) {
+            const int cpt = gpi == 2 ? UC / 2 : UC << ish;  // chunks per group
+            for (int g0i = 0; g0i < ng; g0i += NTC) {      // warp-uniform rounds
+                const int gi = g0i + tid;
+                const bool has = gi < ng;
+                const uint32_t slot = has ? gl[gi] : 0u;
+                const int tl = gpi == 2 ? (int)((slot >> 1) % NTC) : (int)(slot % NTC);
+                const int itg = gpi == 2 ? (int)((slot >> 1) / NTC) : (int)((slot / NTC) << ish);
+                const int ub = gpi == 2 ? (int)(slot & 1u) * (UC / 2) : 0;
+                for (int q0 = 0; q0 < cpt; q0 += 4) {
+                    uint4 dat[4];
+                    int cc[4];
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        const int q = q0 + h;
+                        const int it = itg + q / UC, u = ub + q % UC;
+                        const int t = it * TPI + u * NWC + (tl >> 5);
+                        cc[h] = -1;
+                        if (has && it < nit && t < ntile) {
+                            const int c = (int)((long long)t * a.pstride % ntile) * TCH + (tl & 31);
+                            if (c < nch) cc[h] = c;
+                        }
+                        dat[h] = cc[h] >= 0 ? ldg16(row + (size_t)cc[h] * 16) : make_uint4(NI, NI, NI, NI);
+                    }
+                    uint32_t hm = 0u;
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        const uint32_t wd[4] = {dat[h].x, dat[h].y, dat[h].z, dat[h].w};
+#pragma unroll
+                        for (int e = 0; e < EPC; ++e) {
+                            const uint32_t bits = (e & 1) ? wd[e >> 1] >> 16 : wd[e >> 1] & 0xFFFFu;
+                            hm |= (uint32_t)(bits - vb < 0x8000u - vb) << (h * EPC + e);
+                        }
+                    }
+                    int at = warp_place(__popc(hm), ctr);
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        uint32_t m8 = (hm >> (h * EPC)) & 0xFFu;
+                        while (m8) {
+                            const int e = __ffs(m8) - 1;
+                            m8 &= m8 - 1u;
+                            put(at, __float_as_uint(chunk_elem<DT>(dat[h], e)) >> 16, (uint32_t)(cc[h] * EPC + e));
+                            ++at;
+                        }
+                    }
+                }
+            }
+            __syncthreads();
+        };
+        auto put_pay = [&](int at, uint32_t bits, uint32_t id) {
+            if (at < PCAP && ACES_IN(at, PCAP)) pay[at] = order_val(fkey(__uint_as_float(bits << 16)), id);
+        };
+        unsigned long long *lst = reinterpret_cast<unsigned long long *>(sk);  // (deferred: the listed ids)
+        bool listed = false, sketch_ok = true;
+        int fb = 1;
+        if (count_on && defer) {
+            // every id >= lim(m) (at most HW - 1 values below the max) is read
+            // back from the groups that reach it, listed and counted
+            const float tl = m - D;
+            uint32_t thc = tl > 0.0f ? (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rd(tl)) : 1u;
+            if (thc < 1u) thc = 1u;
+            if (km - thc > (uint32_t)(HW - 1)) thc = km - (uint32_t)(HW - 1);
+            thb0 = thc;
+            uint32_t *gl = reinterpret_cast<uint32_t *>(pay);
+            const int ng = compact(0x8000u + thc, gl);
+            if (ng <= GCAP) {
+                sketch_ok = false;  // (the list takes its place)
+                reread(gl, ng, thc, &s_nrec, [&](int at, uint32_t bits, uint32_t id) {
+                    if (at < LIST_BF && ACES_IN(at, LIST_BF)) lst[at] = order_val(fkey(__uint_as_float(bits << 16)), id);
+                    if (ACES_IN(bits - thb0, HW)) atomicAdd(&hist[bits - thb0], 1u);
+                });
+                listed = s_nrec <= LIST_BF;
+                fb = scan(thc);
+            }
+        } else if (count_on && km < thb0 + HW) {
+            fb = scan(lim_of(m));
+        }
+        if (fb == 1) {
+            // the crossing (or the row max) lies outside the counted values:
+            // a second pass counts the row again, from the row max down as far
+            // as the window reaches
+            thb0 = km > (uint32_t)(HW - 1) ? km - (uint32_t)(HW - 1) : 1u;
+            for (int i = tid; i < HW; i += NTC) hist[i] = 0u;
+            __syncthreads();
+            const uint32_t span = km + 1u - thb0;
+            for (int c0 = 0; c0 < nch; c0 += NTC * UC) {
+#pragma unroll
+                for (int u = 0; u < UC; ++u) {
+                    const int c = c0 + u * NTC + tid;
+                    w[u] = c < nch ? ldg16(row + (size_t)c * 16) : make_uint4(NI, NI, NI, NI);
+                }
+#pragma unroll
+                for (int u = 0; u < UC; ++u) {
+                    const uint32_t wd[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint32_t lo = (wd[q] & 0xFFFFu) - thb0, hi = (wd[q] >> 16) - thb0;
+                        if (lo < span && ACES_IN(lo, HW)) atomicAdd(&hist[lo], 1u);
+                        if (hi < span && ACES_IN(hi, HW)) atomicAdd(&hist[hi], 1u);
+                    }
+                }
+            }
+            __syncthreads();
+            if (tid == 0) atomicAdd(&a.ws.fb_count[10], 1);
+            fb = scan(thb0);
+            listed = false;
+        }
+        if (fb != 0) {
+            if (tid == 0) fallback_row(a, r, m, kref, S);
+            return;
+        }
+        L = s_L;
+        const int vs = s_vs, j = s_j, vr = s_vk;
+        const uint32_t vsb = thb0 + (uint32_t)vs;  // crossing value (bit pattern)
+        const bool exact = !all_in && vr == vs;    // every id of the crossing value is read below
+        if (vr >= 0) {
+            // ---- the ids at or above value vr, then ordered ----
+            const uint32_t vrb = thb0 + (uint32_t)vr;  // its bit pattern
+            if (listed) {
+                const unsigned long long omin = (unsigned long long)fkey(__uint_as_float(vrb << 16)) << 32;
+                const int nlst = s_nrec;
+                for (int i0 = 0; i0 < nlst; i0 += NTC) {  // warp-uniform rounds
+                    const int i = i0 + tid;
+                    const unsigned long long o = i < nlst ? lst[i] : 0ull;
+                    const bool take = i < nlst && o >= omin;
+                    const int at = warp_place(take ? 1 : 0, &s_npay);
+                    if (take && at < PCAP && ACES_IN(at, PCAP)) pay[at] = o;
+                }
+                __syncthreads();
+            } else if (sketch_ok) {
+                const int ng = compact(0x8000u + vrb, glist);
+                if (ng > GCAP) {
+                    if (tid == 0) fallback_row(a, r, m, kref, S);
+                    return;
+                }
+                reread(glist, ng, vrb, &s_npay, put_pay);
+            } else {
+                // (the sketch was overwritten) one more pass over the row
+                for (int c0 = 0; c0 < nch; c0 += NTC * 4) {
+                    uint4 dat[4];
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        const int c = c0 + h * NTC + tid;
+                        dat[h] = c < nch ? ldg16(row + (size_t)c * 16) : make_uint4(NI, NI, NI, NI);
+                    }
+                    uint32_t hm = 0u;
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        const uint32_t wd[4] = {dat[h].x, dat[h].y, dat[h].z, dat[h].w};
+#pragma unroll
+                        for (int e = 0; e < EPC; ++e) {
+                            const uint32_t bits = (e & 1) ? wd[e >> 1] >> 16 : wd[e >> 1] & 0xFFFFu;
+                            hm |= (uint32_t)(bits - vrb < 0x8000u - vrb) << (h * EPC + e);
+                        }
+                    }
+                    int at = warp_place(__popc(hm), &s_npay);
+#pragma unroll
+                    for (int h = 0; h < 4; ++h) {
+                        uint32_t m8 = (hm >> (h * EPC)) & 0xFFu;
+                        while (m8) {
+                            const int e = __ffs(m8) - 1;
+                            m8 &= m8 - 1u;
+                            put_pay(at, __float_as_uint(chunk_elem<DT>(dat[h], e)) >> 16,
+                                    (uint32_t)((c0 + h * NTC + tid) * EPC + e));
+                            ++at;
+                        }
+                    }
+                }
+                __syncthreads();
+            }
+            const int npay = s_npay;
+            if (npay != s_nge) {  // (cannot happen: the counts and the ids agree)
+                if (tid == 0) fallback_row(a, r, m, kref, S);
+                return;
+            }
+            // order them (descending order value)
+            if (npay <= RANK_MAX) {
+                ord = sorted;
+                for (int i = tid; i < npay; i += NTC) {
+                    const unsigned long long key = pay[i];
+                    int rank = 0;
+#pragma unroll 4
+                    for (int t = 0; t < npay; ++t) rank += pay[t] > key;
+                    if (ACES_IN(rank, PCAP)) ord[rank] = key;
+                }
+            } else {
+                if (tid == 0) atomicAdd(&a.ws.fb_count[3], 1);
+                ord = pay;
+                const int np = next_pow2(npay);
+                for (int i = npay + tid; i < np; i += NTC)
+                    if (ACES_IN(i, PCAP)) pay[i] = 0ull;
+                __syncthreads();
+                bitonic_sort_desc(pay, np);
+            }
+            __syncthreads();
+        }
+        const int n_nuc = s_nnuc;
+        if (tid == 0) {
+            if (all_in) {
+                s_cut = 0ull;
+            } else if (exact) {
+                s_cut = ord[n_nuc - 1];
+            } else {
+                s_cut = ((unsigned long long)fkey(val16(0x8000u + vsb)) << 32) | (unsigned long long)(uint32_t)j;
+                atomicAdd(&a.ws.fb_count[5], 1);
+            }
+            s_zx = zx;
+            s_xb = xb;
+        }
+        // keep the nucleus for the residual step when it fits
+        if (exact && a.ws.nuc != nullptr && n_nuc <= NUC_CAP) {
+            for (int i = tid; i < n_nuc; i += NTC)
+                if (ACES_IN(i, NUC_CAP)) a.ws.nuc[(size_t)r * NUC_CAP + i] = ord[i];
+            nnuc = n_nuc;
+        }
+        lazy = !all_in && !exact;
+        __syncthreads();
+        // the draft token's value equals the crossing value and that value's
+        // ids were not read: its rank among them (ids below it) decides
+        if (lazy && s_xb >= 0 && s_xb < a.V && key16(__float_as_uint(s_zx) >> 16) == 0x8000u + vsb) {
+            const int xr = s_xb;
+            const float vsv = val16(0x8000u + vsb);
+            const __nv_bfloat162 v2 = __floats2bfloat162_rn(vsv, vsv);
+            uint32_t cnt = 0u;
+            for (int cc = tid; cc * EPC < xr; cc += NTC) {
+                const uint4 wv = ldg16(row + (size_t)cc * 16);
+                const uint32_t wd[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint32_t mk = __heq2_mask(*reinterpret_cast<const __nv_bfloat162 *>(&wd[q]), v2);
+                    const int x0 = cc * EPC + 2 * q;
+                    cnt += ((mk & 1u) && x0 < xr) + ((mk >> 16 & 1u) && x0 + 1 < xr);
+                }
+            }
+            const unsigned long long below = block_reduce_n<NTC>((unsigned long long)cnt, s_redu, SumU64());
+            if (tid == 0) {
+                atomicAdd(&a.ws.fb_count[7], 1);
+                // x~ is in the nucleus iff fewer than j ids of its value precede it
+                zx = below < (unsigned long long)j ? vsv : -INFINITY;
+            }
+        }
+        v_need = all_in ? (L > 0 ? order_value(ord[L - 1]) : m) : val16(0x8000u + vsb);
+        if (tid == 0) atomicAdd(&a.ws.fb_count[2], 1);
+    } else {
+        // ================= float32: list mode =================
+        // Chunks holding an id >= the capture threshold are recorded (16-byte
+        // chunk and index).  Hinted rows: the threshold is the running max
+        // minus D, so at the end every id >= (row max - D) was recorded.
+        // The first rows: the sample's ids within NSB bins of its max are
+        // binned; the bins where the sample's mass (from the exact exp-sums)
+        // reaches top_p and where its count reaches nmin set a fixed
+        // threshold.
+        float thlo = INFINITY;
+        if (!hinted) {
+            if (have) {
+#pragma unroll
+                for (int u = 0; u < UC; ++u) {
+                    const float cmx = max2_value<DT>(chunk_max2<DT>(w[u]));
+                    if (!__any_sync(0xffffffffu, (m1 - cmx) * a.inv_ws < (float)NSB)) continue;
+#pragma unroll 1  // (unrolled, the independent atomics spill registers)
+                    for (int e = 0; e < EPC; ++e) {
+                        const float d = (m1 - chunk_elem<DT>(w[u], e)) * a.inv_ws;
+                        if (d < (float)NSB && ACES_IN((int)d, NSB)) atomicAdd(&sbin[wid][(int)d], 1u);
+                    }
+                }
+            }
+            // the sample's mass in units of 2^((z - m1) c)
+            {
+                const float kw = warp_max(k_t);
+                float sw = (s_t + e_t) * pow2_int(fmaxf(k_t - kw, -1000.0f));
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) sw += __shfl_xor_sync(0xffffffffu, sw, o);
+                if (lane == 0) redh[wid] = have ? sw * ex2(kw - m1 * a.c) : 0.0f;
+            }
+            __syncthreads();
+            if (wid == 0 && have) {
+                uint32_t c0 = 0u, c1 = 0u;
+                float M = 0.0f;
+#pragma unroll
+                for (int i = 0; i < NWC; ++i) {
+                    if (2 * lane < NSB) c0 += sbin[i][2 * lane];
+                    if (2 * lane + 1 < NSB) c1 += sbin[i][2 * lane + 1];
+                    M += redh[i];
+                }
+                constexpr float L2B = 1.4426950408889634f / SPB;
+                const float ms0 = (float)c0 * ex2(-(2 * lane + 0.5f) * L2B), ms1 = (float)c1 * ex2(-(2 * lane + 1.5f) * L2B);
+                float pm = ms0 + ms1;
+                uint32_t pc = c0 + c1;
+                for (int o = 1; o < 32; o <<= 1) {
+                    const float tm = __shfl_up_sync(0xffffffffu, pm, o);
+                    const uint32_t tc = __shfl_up_sync(0xffffffffu, pc, o);
+                    if (lane >= o) {
+                        pm += tm;
+                        pc += tc;
+                    }
+                }
+                const float pm0 = pm - ms1, pc0f = (float)(pc - c1);  // cumulative through bin 2*lane
+                const float f = a.samp_frac;
+                // first bin whose cumulative reaches a target (NSB when none)
+                auto first_bin = [&](bool h0, bool h1) -> int {
+                    const int hb = h0 ? 2 * lane : (h1 ? 2 * lane + 1 : NSB);
+                    const unsigned bal = __ballot_sync(0xffffffffu, hb < NSB);
+                    return bal ? __shfl_sync(0xffffffffu, hb, __ffs(bal) - 1) : NSB;
+                };
+                auto bin_of_count = [&](float n) { return first_bin(pc0f >= n * f, (float)pc >= n * f); };
+                int blo;
+                if (all_in) {
+                    blo = bin_of_count((float)a.nmin);
+                } else {
+                    const float tm = a.top_p * M;
+                    const int bx = first_bin(pm0 >= tm, pm >= tm);
+                    blo = max(bx + MARGIN_BINS, bin_of_count((float)a.nmin));
+                }
+                blo = min(blo, NSB - 1);
+                if (lane == 0) s_thlo = m1 - (float)(blo + 1) * (a.T / SPB);
+            }
+            __syncthreads();
+            if (have) thlo = s_thlo;
+        }
+        // records the chunks in hb (those holding an id >= the capture
+        // threshold): one vote per iteration, one warp-aggregated atomic per
+        // chunk position that has any; the ids are extracted after the stream
+        auto record_hits = [&](uint32_t hb) {
+            if (!__any_sync(0xffffffffu, hb != 0u)) return;
+            int tile = tile0;
+#pragma unroll
+            for (int u = 0; u < UC; ++u) {
+                const bool hit = (hb >> u) & 1u;
+                const unsigned bal = __ballot_sync(0xffffffffu, hit);
+                if (bal != 0u) {
+                    const int lead = __ffs(bal) - 1;
+                    int base = 0;
+                    if (lane == lead) base = atomicAdd(&s_nrec, __popc(bal));
+                    base = __shfl_sync(0xffffffffu, base, lead);
+                    if (hit) {
+                        const int at = base + __popc(bal & ((1u << lane) - 1u));
+                        if (at < CREC && ACES_IN(at, CREC)) {
+                            rec_dat[at] = w[u];
+                            rec_idx[at] = (uint32_t)(tile * TCH + lane);
+                        }
+                    }
+                }
+                tile += a.pstride_w;
+                if (tile >= ntile) tile -= ntile;
+            }
+        };
+        {
+            float th = hinted ? m1 - D : thlo;
+            uint32_t hb = mask_of(th);  // (iteration 0 is loaded and summed)
+            for (int it = 0; it < nit; ++it) {
+                if (it > 0) {
+                    tile0 += a.pstride_it;
+                    if (tile0 >= ntile) tile0 -= ntile;
+                    load(it);
+                    if (hinted) th = running_max() - D;
+                    hb = math(th, im, g0, g1);
+                    if (hinted) publish_max(im);
+                }
+                record_hits(hb);
+            }
+        }
+        if (finish_sums()) return;
+        const int nrec = s_nrec;
+        if (a.force_fb || nrec > CREC) {
+            if (tid == 0) fallback_row(a, r, m, kref, S);
+            return;
+        }
+        const float thc = hinted ? m - D : thlo;  // every id >= thc was recorded
+        // expand the records: the ids >= thc of every recorded chunk (all such
+        // ids lie in recorded chunks), as 64-bit order values
         if (tid == 0) s_nl = 0;
         __syncthreads();
         for (int i0 = 0; i0 < nrec; i0 += NTC) {  // warp-uniform rounds
@@ -648,23 +1198,16 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
 #pragma unroll
             for (int e = 0; e < EPC; ++e) {
                 const float v = Elem<DT>::get(dat, e);
-                append_cap(list, &s_nl, in && v >= th, order_val(fkey(v), base + (uint32_t)e), LCAP);
+                append_cap(list, &s_nl, in && v >= thc, order_val(fkey(v), base + (uint32_t)e), LCAP);
             }
         }
         __syncthreads();
-    }
-    const int nl = s_nl;
-    if (nl > LCAP) {
-        if (tid == 0) fallback_row(a, r, m, kref, S);
-        return;
-    }
-    const unsigned long long tg = all_in ? 0ull : (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
-    unsigned long long *ord;  // the first ids of the nucleus in order (at least the payload)
-    int lazy = 0;
-    int nnuc = -1;            // nucleus ids written to the row's list (-1: none)
-
-    if (mode == 0) {
-        // ================= list mode =================
+        const int nl = s_nl;
+        if (nl > LCAP) {
+            if (tid == 0) fallback_row(a, r, m, kref, S);
+            return;
+        }
+        const unsigned long long tg = all_in ? 0ull : (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
         // counts of the listed ids in bins of T/8 below m; a bin's ids each
         // carry at least its lower edge's mass, so the first bin where that
         // lower bound of the cumulative mass reaches the target holds or
@@ -845,196 +1388,17 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         if (nnuc > 0)
             for (int i = tid; i < nnuc; i += NTC)
                 if (ACES_IN(i, NUC_CAP)) a.ws.nuc[(size_t)r * NUC_CAP + i] = ord[i];
-    } else {
-        // ================= value mode (bfloat16) =================
-        const uint32_t thk = key16(__float_as_uint(thlo) >> 16);
-        const uint32_t km = key16(__float_as_uint(m) >> 16);
-        if (km - thk >= (uint32_t)HW) {  // ids above the window were not counted
-            if (tid == 0) fallback_row(a, r, m, kref, S);
-            return;
-        }
-        if (tid == 0) atomicAdd(&a.ws.fb_count[2], 1);
-        // prefix scan over the values, highest first, four per thread
-        constexpr int PERV = HW / NTC;
-        const int d0 = tid * PERV;  // values thk + HW - 1 - d0 - i
-        auto vmass = [&](int i, uint32_t cn) -> unsigned long long {
-            return cn ? (unsigned long long)cn * id_fx(val16(thk + (uint32_t)(HW - 1 - d0 - i)), a.c, kref) : 0ull;
-        };
-        uint32_t cnv[PERV];
-        unsigned long long bm = 0ull, bc = 0ull;
-#pragma unroll
-        for (int i = 0; i < PERV; ++i) {
-            cnv[i] = hist[HW - 1 - d0 - i];
-            bm += vmass(i, cnv[i]);
-            bc += cnv[i];
-        }
-        if (tid == 0) {
-            s_vs = -1;
-            s_vk = -1;
-        }
-        unsigned long long mtot, ctot;
-        const unsigned long long mex = block_exscan_n<NTC>(bm, s_redu, &mtot);
-        const unsigned long long cex = block_exscan_n<NTC>(bc, s_redu, &ctot);
-        {
-            unsigned long long cmv = mex, ccv = cex;
-#pragma unroll
-            for (int i = 0; i < PERV; ++i) {
-                const unsigned long long mm = vmass(i, cnv[i]);
-                if (cnv[i] && cmv < tg && cmv + mm >= tg) {
-                    const unsigned long long e1 = mm / cnv[i];
-                    s_vs = HW - 1 - d0 - i;
-                    s_above = cmv;
-                    s_cab = ccv;
-                    s_j = (int)((tg - cmv + e1 - 1) / e1);
-                }
-                cmv += mm;
-                ccv += cnv[i];
-            }
-        }
-        __syncthreads();
-        if (s_vs < 0) {  // the counted ids hold too little mass
-            if (tid == 0) fallback_row(a, r, m, kref, S);
-            return;
-        }
-        const unsigned long long n_nuc = s_cab + (unsigned long long)s_j;
-        const int L = (int)(n_nuc < (unsigned long long)a.k ? n_nuc : (unsigned long long)a.k);
-        if (L > 0) {
-            unsigned long long ccv = cex;
-#pragma unroll
-            for (int i = 0; i < PERV; ++i) {
-                if (ccv < (unsigned long long)L && ccv + cnv[i] >= (unsigned long long)L) s_vk = HW - 1 - d0 - i;
-                ccv += cnv[i];
-            }
-        }
-        if (tid == 0) {
-            s_npay = 0;
-            s_ntie = 0;
-            s_nn = 0;
-        }
-        __syncthreads();
-        const uint32_t vsk = thk + (uint32_t)s_vs;                       // crossing value's key
-        const uint32_t vkk = L > 0 ? thk + (uint32_t)s_vk : 0xFFFFFFFFu;  // last payload value's key
-        const uint32_t tpk = key16(__float_as_uint(thpay) >> 16);
-        if (L > 0 && vkk < tpk) {  // payload ids below the listed range
-            if (tid == 0) fallback_row(a, r, m, kref, S);
-            return;
-        }
-        const bool exact = vsk >= tpk;  // the crossing value's ids are listed
-        const bool keep = exact && a.ws.nuc != nullptr && n_nuc <= (unsigned long long)NUC_CAP;
-        unsigned long long *pay = work, *tie = work + PCAP;
-        for (int i0 = 0; i0 < nl; i0 += NTC) {  // warp-uniform rounds
-            const int i = i0 + tid;
-            unsigned long long o = 0ull;
-            uint32_t kk = 0u;
-            if (i < nl) {
-                o = list[i];
-                kk = key16(__float_as_uint(order_value(o)) >> 16);
-            }
-            const bool in = i < nl;
-            append_cap(pay, &s_npay, in && kk >= vkk, o, PCAP);
-            append_cap(tie, &s_ntie, in && exact && kk == vsk, o, PCAP);
-            if (keep) {  // nucleus ids above the crossing value
-                const bool tk = in && kk > vsk;
-                const unsigned bal = __ballot_sync(0xffffffffu, tk);
-                if (bal) {
-                    int base = 0;
-                    if (lane == __ffs(bal) - 1) base = atomicAdd(&s_nn, __popc(bal));
-                    base = __shfl_sync(0xffffffffu, base, __ffs(bal) - 1);
-                    const int at = base + __popc(bal & ((1u << lane) - 1u));
-                    if (tk && ACES_IN(at, NUC_CAP)) a.ws.nuc[(size_t)r * NUC_CAP + at] = o;
-                }
-            }
-        }
-        __syncthreads();
-        const int npay = s_npay, ntie = s_ntie;
-        if (npay > PCAP || ntie > PCAP) {
-            if (tid == 0) fallback_row(a, r, m, kref, S);
-            return;
-        }
-        // rank: the first L payload ids go to ord (the list is no longer
-        // needed), the crossing value's id of rank j - 1 is the cut
-        ord = list;
-        const int LL = L < npay ? L : npay;
-        for (int i = tid; i < npay; i += NTC) {
-            const unsigned long long key = pay[i];
-            int rank = 0;
-#pragma unroll 4
-            for (int t = 0; t < npay; ++t) rank += pay[t] > key;
-            if (rank < LL && ACES_IN(rank, LCAP)) ord[rank] = key;
-        }
-        const int j = s_j;
-        if (exact) {
-            const int nb = s_nn;
-            for (int i = tid; i < ntie; i += NTC) {
-                const unsigned long long key = tie[i];
-                int rank = 0;
-#pragma unroll 4
-                for (int t = 0; t < ntie; ++t) rank += tie[t] > key;
-                if (rank == j - 1) s_cut = key;
-                if (keep && rank < j && ACES_IN(nb + rank, NUC_CAP)) a.ws.nuc[(size_t)r * NUC_CAP + nb + rank] = key;
-            }
-        }
-        if (keep) nnuc = (int)n_nuc;
-        // exact sum of the payload masses, for the tail
-        unsigned long long loc = 0ull;
-        __syncthreads();
-        for (int i = tid; i < LL; i += NTC) loc += id_fx(order_value(ord[i]), a.c, kref);
-        const unsigned long long cumL = block_reduce_n<NTC>(loc, s_redu, SumU64());
-        if (tid == 0) {
-            const float vsv = val16(vsk);
-            const unsigned long long es = id_fx(vsv, a.c, kref);
-            const unsigned long long snfx = s_above + (unsigned long long)j * es;
-            s_Snuc = (double)snfx * FX_INV;
-            s_inv_S = inv_mass(s_Snuc);
-            s_cumL_fx = cumL;
-            s_L = LL;
-            if (!exact) {
-                s_cut = ((unsigned long long)fkey(vsv) << 32) | (unsigned long long)(uint32_t)j;
-                atomicAdd(&a.ws.fb_count[5], 1);
-            }
-            s_zx = zx;
-            s_xb = xb;
-        }
-        lazy = !exact;
-        __syncthreads();
-        // the draft token's value equals the crossing value and that value's
-        // ids were not listed: its rank among them (ids below it) decides
-        if (lazy && s_xb >= 0 && s_xb < a.V && key16(__float_as_uint(s_zx) >> 16) == vsk) {
-            const int xr = s_xb;
-            const __nv_bfloat162 v2 = __floats2bfloat162_rn(val16(vsk), val16(vsk));
-            uint32_t cnt = 0u;
-            for (int cc = tid; cc * EPC < xr; cc += NTC) {
-                const uint4 wv = ldg16(row + (size_t)cc * 16);
-                const uint32_t wd[4] = {wv.x, wv.y, wv.z, wv.w};
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint32_t mk = __heq2_mask(*reinterpret_cast<const __nv_bfloat162 *>(&wd[q]), v2);
-                    const int x0 = cc * EPC + 2 * q;
-                    cnt += ((mk & 1u) && x0 < xr) + ((mk >> 16 & 1u) && x0 + 1 < xr);
-                }
-            }
-            const unsigned long long below = block_reduce_n<NTC>((unsigned long long)cnt, s_redu, SumU64());
-            if (tid == 0) {
-                atomicAdd(&a.ws.fb_count[7], 1);
-                // x~ is in the nucleus iff fewer than j ids of its value precede it
-                s_zx = below < (unsigned long long)j ? 1.0f : 0.0f;
-            }
-            __syncthreads();
-            if (tid == 0) zx = s_zx > 0.0f ? val16(vsk) : -INFINITY;  // in: keep its value; out: mass 0
-        }
+
+        L = s_L;
+        v_need = all_in ? (L > 0 ? order_value(ord[L - 1]) : m) : order_value(s_cut);
     }
     // ---- outputs ----
-    const int L = s_L;
-    if (tid == 0) {  // publish the depths this row needed, for later rows
-        const float vx = all_in ? m : (lazy ? fkey_inv((uint32_t)(s_cut >> 32)) : order_value(s_cut));
-        const float vl = L > 0 ? order_value(ord[L - 1]) : m;
-        const float m1s = s_m1;  // the sample max (written by the estimate, which ran: no fallback here)
-        const float dxf = (m1s - vx) * a.inv_ws, dkf = (m1s - vl) * a.inv_ws;
-        const int dx = all_in ? 0 : (dxf > 0.0f ? (int)fminf(dxf, (float)(NSB - 1)) : 0);
-        const int dk = dkf > 0.0f ? (int)fminf(dkf, (float)(NSB - 1)) : 0;
-        const int dd = max(dx, dk);
-        if (ACES_IN(dd, NSB)) atomicAdd(&a.ws.fb_count[WS_DEPTH0 + dd], 1);
+    if (tid == 0) {  // publish the depth this row needed, for later rows
+        const float dxf = (m - v_need) * a.inv_ws;
+        const int dx = dxf > 0.0f ? (int)fminf(dxf, (float)(NSB - 1)) : 0;
+        if (ACES_IN(dx, NSB)) atomicAdd(&a.ws.fb_count[WS_DEPTH + dx], 1);
         atomicAdd(&a.ws.fb_count[8], 1);
+        if (hinted) atomicAdd(&a.ws.fb_count[9], 1);
     }
     const float inv_S = s_inv_S;
     for (int j = tid; j < a.k; j += NTC) {
@@ -1121,14 +1485,23 @@ void rows_cap_layout(RowArgs &a, int dt) {
                 break;
             }
     a.inv_ws = (float)(SPB / (double)a.T);
-    a.nmin = 4 * a.k > 256 ? 4 * a.k : 256;
-    a.npay = 4 * a.k > 64 ? 4 * a.k : 64;
+    a.nmin = 2 * a.k + 64 > 256 ? 2 * a.k + 64 : 256;
+    // sketch groups: 4 chunks (two per thread and iteration) when they fit,
+    // else 8 chunks of 2^sk_ish iterations
+    const int nit = (ntile + TPI - 1) / TPI;
+    a.sk_gpi = 2;
+    a.sk_ish = 0;
+    if ((long long)nit * NTC * 2 > SKG) {
+        a.sk_gpi = 1;
+        while ((long long)((nit + (1 << a.sk_ish) - 1) >> a.sk_ish) * NTC > SKG) ++a.sk_ish;
+    }
 }
 
 // The dynamic shared memory above 48 KB needs an opt-in per device, set
 // once per device on the first launch there (outside any stream capture).
 template <int DT>
 static cudaError_t launch_cap_dt(const RowArgs &a, cudaStream_t s) {
+    constexpr int smem = DT == ACES_BF16 ? SMEM_BF : SMEM_F32;
     static std::mutex mu;
     static bool ready[64];
     int dev = 0;
@@ -1136,12 +1509,12 @@ static cudaError_t launch_cap_dt(const RowArgs &a, cudaStream_t s) {
     {
         std::lock_guard<std::mutex> lock(mu);
         if (!ready[dev]) {
-            const cudaError_t e = cudaFuncSetAttribute(k_rows_cap<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize, CAP_SMEM);
+            const cudaError_t e = cudaFuncSetAttribute(k_rows_cap<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
             if (e != cudaSuccess) return e;
             ready[dev] = true;
         }
     }
-    k_rows_cap<DT><<<(unsigned)a.rows, NTC, CAP_SMEM, s>>>(a);
+    k_rows_cap<DT><<<(unsigned)a.rows, NTC, smem, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -1,12 +1,14 @@
 """Parity on inputs built to drive each branch of the row kernels.
 
-The workspace's first eight int32 words count, per call: rows handed to the
-exact general kernel, bounded-wait timeouts (reserved), rows the single-pass
-kernel captured by value histogram, rows whose candidates were ordered by
-bitonic sort (more than 512), rows the general kernel finished by radix
-selection, rows whose nucleus cut was left to the resolve step, rows the
-general kernel finished by its bfloat16 value histogram, and accept tests
-that ranked the draft token among the ids of the crossing value.  Each test
+The workspace's first ten int32 words count, per call: rows handed to the
+exact general kernel, bounded-wait timeouts (reserved), bfloat16 rows the
+single-pass kernel finished from its value counts, rows whose candidates were
+ordered by bitonic sort (more than 512), rows the general kernel finished by
+radix selection, rows whose nucleus cut was left to the resolve step, rows
+the general kernel finished by its bfloat16 value histogram, accept tests
+that ranked the draft token among the ids of the crossing value, rows that
+published their depth, rows that took their depth from finished rows, and
+rows whose values were counted in a second pass.  Each test
 asserts the branch it targets was taken, then compares every output with the
 float64 oracle under the rules of tests/parity.py.  Tests of the general
 kernel's own branches call the exact entry point (every row on that kernel).
@@ -24,7 +26,7 @@ pytestmark = pytest.mark.gpu
 
 torch = pytest.importorskip("torch")
 
-FALLBACK, TIMEOUTS, VALUE_MODE, BITONIC, RADIX, LAZY, GEN_VALHIST, TIE_RANK = range(8)
+FALLBACK, TIMEOUTS, VALUE_MODE, BITONIC, RADIX, LAZY, GEN_VALHIST, TIE_RANK, PUBLISHED, HINTED, RECOUNT = range(11)
 
 
 @pytest.fixture(scope="module")
@@ -49,7 +51,7 @@ def _run(A, orc, w, z, exact=False, inp=None):
     g = A.verify(zt, q, xt, u, w.T, w.top_p, w.k, workspace=ws, exact=exact)
     torch.cuda.synchronize()
     g = {key: v.cpu().numpy() for key, v in g.items()}
-    counters = ws[:32].view(torch.int32).cpu().numpy().tolist()
+    counters = ws[:64].view(torch.int32).cpu().numpy().tolist()
     o = orc.verify(z, inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
     res = parity.compare_verify(inp, g, o, w.top_p, z.dtype == np.uint16, w.k)
     return counters, res
@@ -79,22 +81,21 @@ def _sampled_ids(V, dtype):
 # the single-pass kernel
 
 
-def test_list_mode_on_the_benchmark_rows(A, orc):
-    # the first 4 sequences of the 256000-id benchmark workload (68 rows, all
-    # estimated from their own sample): small nuclei, listed on chip; a row
-    # whose sample misleads goes to the exact kernel, which is rare
+def test_value_counts_on_the_benchmark_rows(A, orc):
+    # the first 4 sequences of the 256000-id benchmark workload (68 rows, the
+    # first rows of a call: D = 10 T): counted per bf16 value, the payload
+    # re-read from the sketch's groups; no row needs the general kernel
     w = dataclasses.replace(gen.WORKLOADS["b256_k16_v256000_bf16"], B=4)
     z = gen.generate(w)["z"]
     counters, res = _run(A, orc, w, z)
-    assert counters[TIMEOUTS] == 0 and counters[VALUE_MODE] == 0 and counters[LAZY] == 0, counters
-    assert counters[FALLBACK] <= 4, counters
+    assert counters[TIMEOUTS] == 0 and counters[FALLBACK] == 0 and counters[VALUE_MODE] == 68, counters
     assert res["checked_seqs"] >= 3
 
 
-def test_value_mode_on_large_nuclei(A, orc):
-    # rows of the 128256-id recipe (nuclei of thousands of ids): counted per
-    # bf16 value while streaming; the crossing value's ids are not listed, so
-    # the cut is left to the resolve step, which finds it for the drawn rows
+def test_large_nuclei_leave_the_cut_to_the_resolve_step(A, orc):
+    # rows of the 128256-id recipe (nuclei of thousands of ids, k = 32): the
+    # crossing value's ids are not among the payload's, so the cut is left to
+    # the resolve step, which finds it for the drawn rows
     w = gen.make_workload(3, 4, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=41)
     z = gen.generate(w)["z"]
     counters, res = _run(A, orc, w, z)
@@ -102,11 +103,11 @@ def test_value_mode_on_large_nuclei(A, orc):
     assert res["checked_seqs"] >= 2
 
 
-def test_value_mode_with_listed_crossing(A, orc):
+def test_exact_cut_when_the_nucleus_fits_the_payload(A, orc):
     # 50 dominant ids at 15 outside the sampled tiles, 60000 ids in [6, 8]:
-    # the sample sees only the bulk, so the capture is deep and counted per
-    # value; the nucleus is the 50 ids, inside the payload list (the 256 ids
-    # the count floor keeps), so the cut is exact on chip
+    # the sample sees only the bulk; the running max reaches 15 later.  The
+    # nucleus (about 35 of the 50 tied ids) is shorter than k, so the payload
+    # re-read holds every id of the crossing value and the cut is exact
     V = 65536
     w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.5, k=64, seed=45)
     rng = np.random.default_rng(45)
@@ -122,10 +123,10 @@ def test_value_mode_with_listed_crossing(A, orc):
     assert res["checked_seqs"] >= 1
 
 
-def test_value_mode_draft_token_on_the_crossing_value(A, orc):
+def test_draft_token_on_the_crossing_value(A, orc):
     # the draft token of every draft row is moved to an id holding that row's
     # crossing value (the n_nuc-th id in order), with q > 0 there: the accept
-    # test ranks it among the ids of that value, which were not listed
+    # test ranks it among the ids of that value, which were not read
     w = gen.make_workload(2, 3, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=46)
     inp = dict(gen.generate(w))
     z = inp["z"]
@@ -147,6 +148,38 @@ def test_value_mode_draft_token_on_the_crossing_value(A, orc):
     counters, res = _run(A, orc, w, z, inp=inp)
     assert counters[TIE_RANK] >= 1 and counters[FALLBACK] == 0, counters
     assert res["checked_seqs"] >= 1
+
+
+def _tied_top(V, n_top, seed):
+    """Rows of n_top ids at 10 spread over the row, the rest at -30."""
+    rng = np.random.default_rng(seed)
+    z = np.full((2, 2, V), -30.0, np.float32)
+    for b in range(2):
+        for i in range(2):
+            z[b, i, rng.choice(V, n_top, replace=False)] = 10.0
+    return _bf16(z)
+
+
+def test_payload_ties_ordered_by_bitonic_sort(A, orc):
+    # 700 ids tied at the top value, top_p = 0.5001 (the crossing, 351 ids
+    # in, is not within 1e-6 of it), k = 64: the crossing value is the
+    # payload's last value, so all 700 of its ids are re-read (more than the
+    # 512 ranked directly: bitonic sort) and the cut is exact
+    V = 65536
+    w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.5001, k=64, seed=51)
+    counters, res = _run(A, orc, w, _tied_top(V, 700, 51))
+    assert counters[FALLBACK] == 0 and counters[BITONIC] == 4 and counters[LAZY] == 0, counters
+    assert res["checked_seqs"] == 2
+
+
+def test_payload_ties_beyond_the_candidate_area_fall_back(A, orc):
+    # 1500 ids tied at the payload's last value: more than the 1024 that the
+    # re-read keeps, so the exact general kernel takes the rows
+    V = 65536
+    w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.5001, k=64, seed=52)
+    counters, res = _run(A, orc, w, _tied_top(V, 1500, 52))
+    assert counters[FALLBACK] == 4, counters
+    assert res["checked_seqs"] == 2
 
 
 def test_bitonic_order_for_many_candidates(A, orc):
@@ -178,11 +211,10 @@ def test_more_candidates_than_the_list_falls_back(A, orc):
     assert res["checked_seqs"] == 2
 
 
-def test_a_misleading_sample_falls_back(A, orc):
+def test_a_misleading_sample_is_still_counted(A, orc):
     # the sampled tiles hold 300 ids near 10 and nothing else; the rest of
-    # the row holds 20000 ids at 5, which carry most of the mass: the
-    # estimate puts theta far above the crossing, the capture holds too
-    # little mass, and the exact general kernel takes the row
+    # the row holds 20000 ids at 5, which carry most of the mass.  The counts
+    # reach 10 T below the running max, so the crossing is found on chip
     V = 65536
     w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.9, k=16, seed=47)
     rng = np.random.default_rng(47)
@@ -194,14 +226,32 @@ def test_a_misleading_sample_falls_back(A, orc):
             z[b, i, rng.choice(samp, 300, replace=False)] = rng.uniform(9.8, 10.0, 300)
             z[b, i, rng.choice(rest, 20000, replace=False)] = 5.0
     counters, res = _run(A, orc, w, _bf16(z))
-    assert counters[FALLBACK] == 4, counters
+    assert counters[FALLBACK] == 0 and counters[VALUE_MODE] == 4, counters
     assert res["checked_seqs"] >= 1
 
 
-def test_value_mode_window_exceeded_falls_back(A, orc):
-    # flat rows in [2, 3] (value mode, theta near 0.5) with one id at 1000
-    # outside the sample: it lies beyond the 1024 counted values above
-    # theta, so the row goes to the exact general kernel
+def test_crossing_below_the_counted_values_is_counted_again(A, orc):
+    # one id at 16 and 60000 ids at 5 (T = 1) carry about equal mass, so the
+    # top_p = 0.9 crossing lies 11 T below the max, beyond D = 10 T: a second
+    # pass counts the row from its max down and finds it (k = 1: the payload
+    # is the top id, the crossing value's ids are left to the resolve step)
+    V = 65536
+    w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.9, k=1, seed=53)
+    rng = np.random.default_rng(53)
+    z = np.full((2, 2, V), -30.0, np.float32)
+    for b in range(2):
+        for i in range(2):
+            z[b, i, rng.choice(V, 60000, replace=False)] = 5.0
+            z[b, i, rng.integers(V)] = 16.0
+    counters, res = _run(A, orc, w, _bf16(z))
+    assert counters[FALLBACK] == 0 and counters[RECOUNT] == 4 and counters[LAZY] == 4, counters
+    assert res["checked_seqs"] >= 1
+
+
+def test_a_max_above_the_value_window_is_counted_again(A, orc):
+    # flat rows in [2, 3] with one id at 1000 outside the sample: it lies
+    # beyond the 1024 counted values (at most 767 below the sample's max);
+    # the second pass anchors the window at the row max
     V = 65536
     w = gen.make_workload(2, 1, V, "bf16", T=1.0, top_p=0.9, k=16, seed=48)
     rng = np.random.default_rng(48)
@@ -210,18 +260,36 @@ def test_value_mode_window_exceeded_falls_back(A, orc):
     z = rng.uniform(2.0, 3.0, size=(2, 2, V)).astype(np.float32)
     z[:, :, far] = 1000.0
     counters, res = _run(A, orc, w, _bf16(z))
-    assert counters[FALLBACK] == 4, counters
+    assert counters[FALLBACK] == 0 and counters[RECOUNT] == 4, counters
     assert res["checked_seqs"] >= 1
 
 
-@pytest.mark.parametrize("dtype,V", [("bf16", 600000), ("f32", 300000), ("f32", 1 << 20)],
-                         ids=["bf16_600k", "f32_300k", "f32_1m"])
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_later_rows_take_their_depth_from_finished_rows(A, orc, dtype):
+    # 1088 rows, more than run at once: rows that start after 32 have
+    # finished take D from those rows' depths (bf16: the counts' lower end;
+    # float32: the capture threshold, running max - D).  Shapes of the
+    # 128256-id and of the 32000-id float32 workloads.
+    if dtype == "bf16":
+        w = gen.make_workload(64, 16, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=54)
+    else:
+        w = gen.make_workload(64, 16, 32000, "f32", sigma=3.0, rho=0.8, T=0.8, top_p=0.9, k=32, seed=54)
+    inp = gen.generate(w)
+    counters, res = _run(A, orc, w, inp["z"], inp=dict(inp))
+    # (float32 rows whose capture overflows the 1536 recorded chunks go to
+    # the exact general kernel)
+    assert counters[HINTED] >= 200 and counters[FALLBACK] <= (8 if dtype == "bf16" else 200), counters
+    assert res["checked_seqs"] >= 32
+
+
+@pytest.mark.parametrize("dtype,V", [("bf16", 600000), ("bf16", 1 << 20), ("f32", 300000), ("f32", 1 << 20)],
+                         ids=["bf16_600k", "bf16_1m", "f32_300k", "f32_1m"])
 def test_large_vocabularies(A, orc, dtype, V):
-    w = gen.make_workload(1, 1, V, dtype, T=0.8, top_p=0.9, k=48, seed=34)
+    w = gen.make_workload(4, 1, V, dtype, T=0.8, top_p=0.9, k=48, seed=34)
     z = gen.generate(w)["z"]
     counters, res = _run(A, orc, w, z)
     assert counters[TIMEOUTS] == 0
-    assert res["checked_seqs"] == 1
+    assert res["checked_seqs"] >= 1
 
 
 # ---------------------------------------------------------------------------
@@ -316,11 +384,12 @@ def test_signed_zeros_on_the_general_path(A, orc):
 
 
 def test_general_radix_path(A, orc):
-    # float32 rows of 5000 tied ids at 0 (the rest at -30), top_p = 0.5: the
-    # crossing bin holds more ids than the binned path collects (2048), so
-    # the radix selection finishes the rows; ties go by id
+    # float32 rows of 5000 tied ids at 0 (the rest at -30), top_p = 0.5001
+    # (the crossing, 2501 ids in, is 1e-4 from it: not flagged): the crossing
+    # bin holds more ids than the binned path collects (2048), so the radix
+    # selection finishes the rows; ties go by id
     V = 32768
-    w = gen.make_workload(2, 1, V, "f32", T=1.0, top_p=0.5, k=16, seed=49)
+    w = gen.make_workload(2, 1, V, "f32", T=1.0, top_p=0.5001, k=16, seed=49)
     rng = np.random.default_rng(49)
     z = np.full((2, 2, V), -30.0, np.float32)
     for b in range(2):
