@@ -44,7 +44,7 @@ VERIFY_KERNELS = ["k_rows_cap", "k_rows_general", "k_resolve_cut", "k_resolve_se
 PATHS = ["rows_on_general_kernel", "timeouts", "rows_value_histogram", "rows_bitonic_order",
          "general_rows_radix", "rows_cut_left_to_resolve", "general_rows_value_histogram",
          "accept_tests_ranked_among_ties", "rows_published_depth", "rows_depth_from_finished_rows",
-         "rows_counted_twice"]
+         "rows_counted_twice", "rows_collected_in_a_second_pass"]
 
 
 # ---------------------------------------------------------------------------

@@ -166,8 +166,13 @@ template <> struct Elem<ACES_BF16> {
     }
 };
 
+// 16 bytes of read-only data, not kept in L1 (streamed once)
 __device__ __forceinline__ uint4 ldg16(const void *p) {
-    return __ldg(reinterpret_cast<const uint4 *>(p));
+    uint4 v;
+    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
 }
 
 // ---------------------------------------------------------------------------
@@ -354,21 +359,21 @@ struct SegSum {
 constexpr int NSEG_MAX = 16;
 constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual step
 
-constexpr int WS_COUNTERS = 512;      // bytes of path counters and depth hints at the start of the workspace
+constexpr int WS_COUNTERS = 256;      // bytes of path counters and depth hints at the start of the workspace
 constexpr int WS_DEPTH = 16;          // first of the 40 depth counters of the row kernel's hints (int index)
 // Workspace layout (all offsets 16-byte aligned)
 struct Workspace {
-    int *fb_count;             // [128] path counters and depth hints, cleared by every call: [0] rows handed to the
+    int *fb_count;             // [64] path counters and depth hints, cleared by every call: [0] rows handed to the
                                //       general kernel, [1] reserved (no kernel waits on another),
-                               //       [2] rows captured by value histogram, [3] rows ordered by
-                               //       bitonic sort, [4] rows the general kernel finished by radix
-                               //       selection, [5] rows whose cut was left to the resolve step,
-                               //       [6] rows the general kernel finished by value histogram,
+                               //       [2] bfloat16 rows finished from their value counts, [3] rows
+                               //       ordered by bitonic sort, [4] rows the general kernel finished
+                               //       by radix selection, [5] rows whose cut was left to the resolve
+                               //       step, [6] rows the general kernel finished by value histogram,
                                //       [7] accept tests that ranked the draft token among ties,
-                               //       [8] rows that published the depths they needed,
-                               //       [16..55] how many rows had their crossing, [64..103] their
-                               //       payload end, at each depth (in sample bins of T/4 below
-                               //       the row's sample max)
+                               //       [8] rows that published the depth they needed, [9] rows that
+                               //       took their depth from finished rows, [10] rows counted again
+                               //       in a second pass, [16..55] how many rows needed each depth
+                               //       (in bins of T/4 below the row max)
     RowStat *stats;            // [rows]
     int *acc;                  // [B*K] accept bits
     int *fb_list;              // [rows]
@@ -490,15 +495,14 @@ struct CacheArgs {
     float *bp;
 };
 
-// first rejection index pi_b (K when every draft token was accepted)
-__device__ __forceinline__ int first_reject(const Workspace &ws, int b, int K) {
-    int pi = K;
-    for (int i = 0; i < K; ++i)
-        if (!ws.acc[(size_t)b * K + i]) {
-            pi = i;
-            break;
-        }
-    return pi;
+// first rejection index pi_b (K when every draft token was accepted), by a
+// whole warp: one load per lane and a vote
+static_assert(ACES_MAX_K <= 32, "one accept bit per lane");
+__device__ __forceinline__ int first_reject_warp(const Workspace &ws, int b, int K) {
+    const int lane = threadIdx.x & 31;
+    const bool rej = lane < K && !ws.acc[(size_t)b * K + lane];
+    const unsigned bal = __ballot_sync(0xffffffffu, rej);
+    return bal ? __ffs(bal) - 1 : K;
 }
 
 struct DrawShared {
@@ -522,8 +526,11 @@ __device__ void draw_from_list(const Workspace &ws, const float *q, const float 
                                unsigned long long *pfx, unsigned long long *red, DrawShared *sh) {
     static_assert(2 * NTH >= NUC_CAP, "two nucleus entries per thread");
     const int tid = threadIdx.x;
+    if (tid < 32) {
+        const int pi0 = first_reject_warp(ws, b, K);
+        if (tid == 0) sh->pi = pi0;
+    }
     if (tid == 0) {
-        sh->pi = first_reject(ws, b, K);
         sh->bad = 0;
         sh->tok = -1;
     }

@@ -126,7 +126,10 @@ __global__ void __launch_bounds__(NTR) k_resolve_cut(ResolveArgs a, int nseg, in
     const int b = blockIdx.x / nseg, sg = blockIdx.x % nseg, tid = threadIdx.x;
     pdl_wait();  // the row kernels are complete
     if (a.ws.fb_count[5] == 0 || a.ws.seqdone[b]) return;  // no cut left open / token already drawn
-    if (tid == 0) s_pi = first_reject(a.ws, b, a.K);
+    if (tid < 32) {
+        const int pi0 = first_reject_warp(a.ws, b, a.K);
+        if (tid == 0) s_pi = pi0;
+    }
     __syncthreads();
     const int r = b * (a.K + 1) + s_pi;
     const RowStat rs = a.ws.stats[r];
@@ -136,6 +139,7 @@ __global__ void __launch_bounds__(NTR) k_resolve_cut(ResolveArgs a, int nseg, in
     const char *zrow = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
     const int x_lo = sg * seglen, x_hi = min(a.V, x_lo + seglen);
     unsigned long long cnt = 0ull;
+#pragma unroll 4
     for (int x0 = x_lo + tid * EPT; x0 < x_hi; x0 += TILE) cnt += __popc(ties_of<DT, VEC>(zrow, x_hi, x0, vkey));
     const unsigned long long tot = block_reduce_n<NTR>(cnt, red, SumU64());
     if (tid == 0) {
@@ -192,8 +196,9 @@ __global__ void __launch_bounds__(NTR) k_resolve_seg(ResolveArgs a, int nseg, in
     const int b = blockIdx.x / nseg, sg = blockIdx.x % nseg, tid = threadIdx.x;
     pdl_wait();  // the row kernels are complete
     if (a.ws.seqdone[b]) return;  // drawn from row pi's nucleus list
+    const int pi0 = tid < 32 ? first_reject_warp(a.ws, b, a.K) : 0;
     if (tid == 0) {
-        const int pi = first_reject(a.ws, b, a.K);
+        const int pi = pi0;
         s_pi = pi;
         s_bad = 0;
         if (sg == 0) a.accept_len[b] = pi;
@@ -213,6 +218,7 @@ __global__ void __launch_bounds__(NTR) k_resolve_seg(ResolveArgs a, int nseg, in
     const int x_lo = sg * seglen, x_hi = min(a.V, x_lo + seglen);
     unsigned long long sr = 0ull, sp = 0ull;
     int bad = 0;
+#pragma unroll 4
     for (int x0 = x_lo + tid * EPT; x0 < x_hi; x0 += TILE) {
         unsigned long long rf[EPT], pf[EPT];
         mass_fx<DT, VEC>(zrow, qrow, x_hi, x0, rs, inv_S, rf, pf, &bad);
@@ -238,8 +244,9 @@ __global__ void __launch_bounds__(NTR) k_resolve_pick(ResolveArgs a, int nseg, i
     const int b = blockIdx.x, tid = threadIdx.x;
     pdl_wait();  // the segment sums are complete
     if (a.ws.seqdone[b]) return;  // drawn from row pi's nucleus list
+    const int pi0 = tid < 32 ? first_reject_warp(a.ws, b, a.K) : 0;
     if (tid == 0) {
-        s_pi = first_reject(a.ws, b, a.K);
+        s_pi = pi0;
         s_tok = -1;
         s_done = 0;
         s_seg = -1;
@@ -338,8 +345,9 @@ __global__ void __launch_bounds__(NTR) k_resolve_pick(ResolveArgs a, int nseg, i
 }
 
 
+// segments of about 8192 ids (four tiles), at most NSEG_MAX per sequence
 int resolve_segments(int V) {
-    int nseg = (V + 32767) / 32768;
+    int nseg = (V + 8191) / 8192;
     return nseg < 1 ? 1 : (nseg > NSEG_MAX ? NSEG_MAX : nseg);
 }
 

@@ -70,8 +70,6 @@ constexpr int HEADROOM = 256;       // of them above the sample's max at least
 constexpr int SKG = 16384;          // sketch entries (group maxima, as 16-bit order keys)
 constexpr int PCAP = 1024;          // ids at or above the payload's last value
 constexpr int GCAP = 1024;          // sketch groups re-read
-constexpr int DEFER_IDS = 768;      // expected ids >= lim(max) below which they are counted after the stream
-constexpr int LIST_BF = SKG / 4;    // ids listed from the re-read groups (in the sketch's area)
 constexpr int SMEM_BF = HW * 4 + SKG * 2 + PCAP * 8;
 // float32
 constexpr int CREC = 1536;          // recorded chunks (16-byte chunk + its index) per row
@@ -263,15 +261,6 @@ __device__ __forceinline__ void fallback_row(const RowArgs &a, int r, float m, f
     a.ws.fb_list[pos] = r;
 }
 
-// the CTA's exp-sum from the per-warp (hi, lo) pairs, in fp64, by warp 0 (a
-// shuffle tree: three dependent fp64 adds instead of eight in one thread)
-__device__ __forceinline__ double warp0_mass(const float *hi, const float *lo, int lane) {
-    double v = lane < NWC ? (double)hi[lane] + (double)lo[lane] : 0.0;
-#pragma unroll
-    for (int o = NWC / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
-}
-
 // appends o to arr[*n] for every lane with take (one atomic per warp); *n
 // may pass cap, entries beyond it are dropped (all lanes of the warp call it)
 __device__ __forceinline__ void append_cap(unsigned long long *arr, int *n, bool take, unsigned long long o, int cap) {
@@ -318,7 +307,7 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     __shared__ float s_thlo, s_zx;
     __shared__ int s_dbins, s_xb;  // s_dbins: D in depth bins (-1: no hints yet)
     __shared__ uint32_t s_mr;  // order key of the running max
-    __shared__ double s_S, s_Snuc;
+    __shared__ double s_Snuc;
     __shared__ float s_inv_S;
     __shared__ unsigned long long s_cut, s_cumL_fx;
     __shared__ unsigned long long s_redu[NWC];
@@ -346,6 +335,8 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     if (tid == 0) {
         s_nrec = 0;
         s_nl = 0;
+        s_fb = 0;
+        s_nstar = INT_MAX;
         s_mr = fkey(-INFINITY);
     }
     // the depths published by the call's finished rows (read by warp 0 only,
@@ -467,23 +458,11 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
             qx = __ldg(a.q + ((size_t)bq * a.K + iq) * a.V + xb);
             ux = __ldg(a.u + (size_t)bq * (a.K + 1) + iq);
         }
+        // each warp: its max, reference kw and exp-sum in units of 2^kw (a
+        // compensated fp32 tree over rescales by exact powers of two)
         {
             const float mw = warp_max(m_t), kw = warp_max(k_t);
-            if (lane == 0) {
-                redf[wid] = mw;
-                redk[wid] = kw;
-            }
-        }
-        __syncthreads();
-        m = redf[0];
-        kref = redk[0];
-#pragma unroll
-        for (int i = 1; i < NWC; ++i) {
-            m = fmaxf(m, redf[i]);
-            kref = fmaxf(kref, redk[i]);
-        }
-        {
-            const float f = pow2_int(fmaxf(k_t - kref, -1000.0f));
+            const float f = pow2_int(fmaxf(k_t - kw, -1000.0f));
             float hi = s_t * f, lo = e_t * f;
             for (int o = 16; o > 0; o >>= 1) {
                 const float h2 = __shfl_xor_sync(0xffffffffu, hi, o);
@@ -494,21 +473,33 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
                 hi = sm;
             }
             if (lane == 0) {
+                redf[wid] = mw;
+                redk[wid] = kw;
                 redh[wid] = hi;
                 redl[wid] = lo;
             }
         }
         __syncthreads();
-        if (wid == 0) {
-            const double Sw = warp0_mass(redh, redl, lane);
-            if (lane == 0) {
-                s_S = Sw;
-                s_fb = 0;
-                s_nstar = INT_MAX;
-            }
+        // every thread combines the warps' parts (fp64, exact rescales)
+        m = redf[0];
+        kref = redk[0];
+#pragma unroll
+        for (int i = 1; i < NWC; ++i) {
+            m = fmaxf(m, redf[i]);
+            kref = fmaxf(kref, redk[i]);
         }
-        __syncthreads();
-        S = s_S;
+        // (fp32 two-sums over exact power-of-two rescales: fp64 is slow here)
+        float sh = 0.0f, sl = 0.0f;
+#pragma unroll
+        for (int i = 0; i < NWC; ++i) {
+            const float f = pow2_int(fmaxf(redk[i] - kref, -1000.0f));  // (an integer <= 0)
+            float sm, er;
+            two_sum(sh, redh[i] * f, sm, er);
+            sl += er + redl[i] * f;
+            sh = sm;
+        }
+        const double Sa = (double)sh + (double)sl;
+        S = Sa;
         if (!(S > 0.0 && S < 1e300) || !(m < INFINITY) || !(kref < 1e30f)) {
             nonfinite_row<NTC>(a, r);
             row_finished(a, r, smem);
@@ -547,11 +538,14 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         // pattern times 4 indexes its counter)
         const uint32_t hbase = (uint32_t)__cvta_generic_to_shared(hist) - thb0 * 4u;
         auto count_hits = [&](uint32_t hb, uint32_t thb) {
-            if (hb == 0u) return;  // (no chunk of this thread reaches thb)
+            // chunk positions where some lane of the warp reaches thb (the
+            // branches are warp-uniform; every lane checks every element)
+            const uint32_t any = __reduce_or_sync(0xffffffffu, hb);
+            if (any == 0u) return;
             const uint32_t span = thb0 + HW - thb;
 #pragma unroll
             for (int u = 0; u < UC; ++u) {
-                if ((hb >> u) & 1u) {
+                if ((any >> u) & 1u) {
                     const uint32_t wd[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
@@ -583,33 +577,7 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
                 }
             }
         };
-        // Rows expected to hold few ids >= lim(m1) (the sample's count,
-        // scaled) defer the counting: the stream only sums and keeps the
-        // sketch, and after it the groups that reach the row's own lim(m)
-        // are read back, their ids listed and counted.  Others count while
-        // streaming.
-        int defer = 0;
-        if (count_on) {
-            const float thf0 = __uint_as_float(lim_of(m1) << 16);
-            uint32_t cnt = 0u;
-#pragma unroll
-            for (int u = 0; u < UC; ++u) cnt += __popc(chunk_hits<DT>(w[u], thf0));
-            cnt = __reduce_add_sync(0xffffffffu, cnt);
-            if (lane == 0) atomicAdd(&s_nl, (int)cnt);
-            __syncthreads();
-            defer = (float)s_nl < (float)DEFER_IDS * a.samp_frac;
-        }
-        if (defer) {
-            for (int it = 0; it < nit; ++it) {
-                if (it > 0) {
-                    tile0 += a.pstride_it;
-                    if (tile0 >= ntile) tile0 -= ntile;
-                    load(it);
-                    math(INFINITY, im, g0, g1);
-                }
-                sketch_put(it);
-            }
-        } else {
+        {
             uint32_t thb = count_on ? lim_of(m1) : 0u;
             float thf = count_on ? __uint_as_float(thb << 16) : INFINITY;
             uint32_t hb = mask_of(thf);  // (iteration 0 is loaded and summed)
@@ -635,7 +603,6 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
             if (tid == 0) fallback_row(a, r, m, kref, S);
             return;
         }
-        const unsigned long long tg = all_in ? 0ull : (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
         auto vmass = [&](int idx) { return id_fx(val16(0x8000u + thb0 + (uint32_t)idx), a.c, kref); };
         unsigned long long *emass = pay;  // (until the re-read) the mass of one id of each counted value
         // ---- the crossing, the payload's end and the values to re-read,
@@ -644,6 +611,8 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         // re-read keeps share the payload's last value ----
         auto scan = [&](uint32_t thc) -> int {
             if (wid == 0) {
+                const unsigned long long tg =
+                    all_in ? 0ull : (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
                 const int top = (int)(km - thb0), lo = (int)(thc - thb0);
                 const int per = (top - lo + 32) >> 5;
                 const int b0 = top - lane * per;  // this lane's values: b0, b0 - 1, ... (>= lo)
@@ -870,29 +839,8 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         auto put_pay = [&](int at, uint32_t bits, uint32_t id) {
             if (at < PCAP && ACES_IN(at, PCAP)) pay[at] = order_val(fkey(__uint_as_float(bits << 16)), id);
         };
-        unsigned long long *lst = reinterpret_cast<unsigned long long *>(sk);  // (deferred: the listed ids)
-        bool listed = false, sketch_ok = true;
         int fb = 1;
-        if (count_on && defer) {
-            // every id >= lim(m) (at most HW - 1 values below the max) is read
-            // back from the groups that reach it, listed and counted
-            const float tl = m - D;
-            uint32_t thc = tl > 0.0f ? (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rd(tl)) : 1u;
-            if (thc < 1u) thc = 1u;
-            if (km - thc > (uint32_t)(HW - 1)) thc = km - (uint32_t)(HW - 1);
-            thb0 = thc;
-            uint32_t *gl = reinterpret_cast<uint32_t *>(pay);
-            const int ng = compact(0x8000u + thc, gl);
-            if (ng <= GCAP) {
-                sketch_ok = false;  // (the list takes its place)
-                reread(gl, ng, thc, &s_nrec, [&](int at, uint32_t bits, uint32_t id) {
-                    if (at < LIST_BF && ACES_IN(at, LIST_BF)) lst[at] = order_val(fkey(__uint_as_float(bits << 16)), id);
-                    if (ACES_IN(bits - thb0, HW)) atomicAdd(&hist[bits - thb0], 1u);
-                });
-                listed = s_nrec <= LIST_BF;
-                fb = scan(thc);
-            }
-        } else if (count_on && km < thb0 + HW) {
+        if (count_on && km < thb0 + HW) {
             fb = scan(lim_of(m));
         }
         if (fb == 1) {
@@ -923,7 +871,6 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
             __syncthreads();
             if (tid == 0) atomicAdd(&a.ws.fb_count[10], 1);
             fb = scan(thb0);
-            listed = false;
         }
         if (fb != 0) {
             if (tid == 0) fallback_row(a, r, m, kref, S);
@@ -936,57 +883,13 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         if (vr >= 0) {
             // ---- the ids at or above value vr, then ordered ----
             const uint32_t vrb = thb0 + (uint32_t)vr;  // its bit pattern
-            if (listed) {
-                const unsigned long long omin = (unsigned long long)fkey(__uint_as_float(vrb << 16)) << 32;
-                const int nlst = s_nrec;
-                for (int i0 = 0; i0 < nlst; i0 += NTC) {  // warp-uniform rounds
-                    const int i = i0 + tid;
-                    const unsigned long long o = i < nlst ? lst[i] : 0ull;
-                    const bool take = i < nlst && o >= omin;
-                    const int at = warp_place(take ? 1 : 0, &s_npay);
-                    if (take && at < PCAP && ACES_IN(at, PCAP)) pay[at] = o;
-                }
-                __syncthreads();
-            } else if (sketch_ok) {
+            {
                 const int ng = compact(0x8000u + vrb, glist);
                 if (ng > GCAP) {
                     if (tid == 0) fallback_row(a, r, m, kref, S);
                     return;
                 }
                 reread(glist, ng, vrb, &s_npay, put_pay);
-            } else {
-                // (the sketch was overwritten) one more pass over the row
-                for (int c0 = 0; c0 < nch; c0 += NTC * 4) {
-                    uint4 dat[4];
-#pragma unroll
-                    for (int h = 0; h < 4; ++h) {
-                        const int c = c0 + h * NTC + tid;
-                        dat[h] = c < nch ? ldg16(row + (size_t)c * 16) : make_uint4(NI, NI, NI, NI);
-                    }
-                    uint32_t hm = 0u;
-#pragma unroll
-                    for (int h = 0; h < 4; ++h) {
-                        const uint32_t wd[4] = {dat[h].x, dat[h].y, dat[h].z, dat[h].w};
-#pragma unroll
-                        for (int e = 0; e < EPC; ++e) {
-                            const uint32_t bits = (e & 1) ? wd[e >> 1] >> 16 : wd[e >> 1] & 0xFFFFu;
-                            hm |= (uint32_t)(bits - vrb < 0x8000u - vrb) << (h * EPC + e);
-                        }
-                    }
-                    int at = warp_place(__popc(hm), &s_npay);
-#pragma unroll
-                    for (int h = 0; h < 4; ++h) {
-                        uint32_t m8 = (hm >> (h * EPC)) & 0xFFu;
-                        while (m8) {
-                            const int e = __ffs(m8) - 1;
-                            m8 &= m8 - 1u;
-                            put_pay(at, __float_as_uint(chunk_elem<DT>(dat[h], e)) >> 16,
-                                    (uint32_t)((c0 + h * NTC + tid) * EPC + e));
-                            ++at;
-                        }
-                    }
-                }
-                __syncthreads();
             }
             const int npay = s_npay;
             if (npay != s_nge) {  // (cannot happen: the counts and the ids agree)

@@ -271,7 +271,7 @@ def test_later_rows_take_their_depth_from_finished_rows(A, orc, dtype):
     # float32: the capture threshold, running max - D).  Shapes of the
     # 128256-id and of the 32000-id float32 workloads.
     if dtype == "bf16":
-        w = gen.make_workload(64, 16, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=54)
+        w = gen.make_workload(96, 16, 128256, "bf16", sigma=3.0, rho=0.5, T=1.0, top_p=0.9, k=32, seed=54)
     else:
         w = gen.make_workload(64, 16, 32000, "f32", sigma=3.0, rho=0.8, T=0.8, top_p=0.9, k=32, seed=54)
     inp = gen.generate(w)
