@@ -36,15 +36,15 @@ sys.path.insert(0, ROOT)
 METRIC = "verified rows/s and achieved HBM GB/s (fraction of GB300 peak) for verify+sparsify"
 WORKLOAD = "b256_k16_v256000_bf16"
 SWEEP_B = (32, 64, 128, 256)
-# kernels of one step: k_rows_cap, k_rows_general, k_resolve_cut,
-# k_resolve_seg, k_resolve_pick (aces_verify), k_cache_build, k_cache_lookup
-KERNELS_PER_STEP = 7
-VERIFY_KERNELS = ["k_rows_cap", "k_rows_general", "k_resolve_cut", "k_resolve_seg", "k_resolve_pick"]
+# kernels of one step: k_rows_cap, k_rows_general, k_resolve_seg,
+# k_resolve_pick (aces_verify), k_cache_build, k_cache_lookup
+KERNELS_PER_STEP = 6
+VERIFY_KERNELS = ["k_rows_cap", "k_rows_general", "k_resolve_seg", "k_resolve_pick"]
 # path counters at the start of the workspace (int32 words)
 PATHS = ["rows_on_general_kernel", "timeouts", "rows_value_histogram", "rows_bitonic_order",
          "general_rows_radix", "rows_cut_left_to_resolve", "general_rows_value_histogram",
          "accept_tests_ranked_among_ties", "rows_published_depth", "rows_depth_from_finished_rows",
-         "rows_counted_twice", "rows_collected_in_a_second_pass"]
+         "rows_counted_twice", "short_rows_published", "rows_sketch_led"]
 
 
 # ---------------------------------------------------------------------------

@@ -351,10 +351,11 @@ __device__ __forceinline__ unsigned long long floor_u_times(float uu, unsigned l
 
 // Exact sums of one vocabulary segment of a sequence's row pi (2^-40 units).
 struct SegSum {
-    unsigned long long r;  // residual max(0, p - q)
-    unsigned long long p;  // p itself
-    int bad;               // a NaN / negative draft probability was seen
-    int pad;
+    unsigned long long r;   // residual max(0, p - q) of the nucleus ids, those of a lazy cut's value aside
+    unsigned long long p;   // p itself, likewise
+    unsigned long long tr;  // residual of the ids of a lazy cut's value
+    int bad;                // a NaN / negative draft probability was seen
+    int nt;                 // ids of a lazy cut's value
 };
 constexpr int NSEG_MAX = 16;
 constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual step
@@ -372,16 +373,16 @@ struct Workspace {
                                //       [7] accept tests that ranked the draft token among ties,
                                //       [8] rows that published the depth they needed, [9] rows that
                                //       took their depth from finished rows, [10] rows counted again
-                               //       in a second pass, [16..55] how many rows needed each depth
-                               //       (in bins of T/4 below the row max)
+                               //       in a second pass, [11] bfloat16 rows that published a short
+                               //       nucleus, [12] rows finished by the sketch-led pass,
+                               //       [16..55] how many rows needed each depth (in bins of T/4
+                               //       below the row max)
     RowStat *stats;            // [rows]
     int *acc;                  // [B*K] accept bits
     int *fb_list;              // [rows]
-    SegSum *seg;               // [B*NSEG_MAX]     (verify only)
+    SegSum *seg;               // [B*NSEG_MAX]     (verify only) cleared by every call
     int *seqcnt;               // [B]              (verify only) rows of the sequence finished by the row kernel
     int *seqdone;              // [B]              (verify only) token already drawn
-    int *cutcnt;               // [B]              (verify only) segments that counted their ties
-    int *tiecnt;               // [B*NSEG_MAX]     (verify only) ties of the cut value per segment
     unsigned long long *nuc;   // [rows*NUC_CAP]   (verify with lists) nucleus order values
 };
 __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
@@ -391,17 +392,17 @@ __host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K, bool lists
     size_t b = WS_COUNTERS + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
                align16((size_t)rows * 4);
     if (K > 0) {
-        b += 3 * align16((size_t)nseq * 4) + align16((size_t)nseq * NSEG_MAX * sizeof(SegSum)) +
-             align16((size_t)nseq * NSEG_MAX * 4);
+        b += 2 * align16((size_t)nseq * 4) + align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
         if (lists) b += (size_t)rows * NUC_CAP * 8;
     }
     return b;
 }
 // bytes at the start of the workspace that every call clears: the counters
-// and, for verification, the per-sequence row counts, done flags and
-// segment counts
+// and, for verification, the per-sequence row counts and done flags and the
+// segment sums (added to atomically)
 __host__ __device__ inline size_t ws_clear_bytes(int nseq, int K) {
-    return WS_COUNTERS + (K > 0 ? 3 * align16((size_t)nseq * 4) : 0);
+    return WS_COUNTERS +
+           (K > 0 ? 2 * align16((size_t)nseq * 4) + align16((size_t)nseq * NSEG_MAX * sizeof(SegSum)) : 0);
 }
 __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K, bool lists) {
     char *p = (char *)base;
@@ -410,15 +411,14 @@ __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, in
     p += WS_COUNTERS;
     w.seqcnt = nullptr;
     w.seqdone = nullptr;
-    w.cutcnt = nullptr;
-    w.tiecnt = nullptr;
+    w.seg = nullptr;
     if (K > 0) {
         w.seqcnt = (int *)p;
         p += align16((size_t)nseq * 4);
         w.seqdone = (int *)p;
         p += align16((size_t)nseq * 4);
-        w.cutcnt = (int *)p;
-        p += align16((size_t)nseq * 4);
+        w.seg = (SegSum *)p;
+        p += align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
     }
     w.stats = (RowStat *)p;
     p += align16((size_t)rows * sizeof(RowStat));
@@ -426,13 +426,8 @@ __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, in
     p += align16((size_t)nseq * K * 4);
     w.fb_list = (int *)p;
     p += align16((size_t)rows * 4);
-    w.seg = nullptr;
     w.nuc = nullptr;
     if (K > 0) {
-        w.seg = (SegSum *)p;
-        p += align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
-        w.tiecnt = (int *)p;
-        p += align16((size_t)nseq * NSEG_MAX * 4);
         if (lists) {
             w.nuc = (unsigned long long *)p;
             p += (size_t)rows * NUC_CAP * 8;

@@ -71,6 +71,15 @@ constexpr int SKG = 16384;          // sketch entries (group maxima, as 16-bit o
 constexpr int PCAP = 1024;          // ids at or above the payload's last value
 constexpr int GCAP = 1024;          // sketch groups re-read
 constexpr int SMEM_BF = HW * 4 + SKG * 2 + PCAP * 8;
+// sketch-led pass: a row is short when at most SHORT_IDS ids reach its
+// crossing (top_p = 1: when k <= SHORT_IDS); later rows take the pass when
+// at least SHORT_NUM / SHORT_DEN of the finished rows were short.  Its areas
+// inside the sketch's (in 8-byte units): the ordered ids [0, 1024), the
+// groups read back and then the kept ids [2048, 3072), the per-value masses
+// [3072, 4096)
+constexpr int SHORT_IDS = 256;
+constexpr int SHORT_NUM = 49, SHORT_DEN = 50;
+constexpr int SK_TMP = 2048, SK_EMASS = 3072;
 // float32
 constexpr int CREC = 1536;          // recorded chunks (16-byte chunk + its index) per row
 constexpr int LCAP = 2048;          // listed ids, expanded from the records after the stream
@@ -80,6 +89,8 @@ constexpr int RANK_MAX = 512;       // ids ordered by direct ranking (more: bito
 static_assert(WS_DEPTH + NSB <= WS_COUNTERS / 4, "the depth histogram fits the counters area");
 static_assert(4 * NUC_CAP * 8 <= SMEM_BF && 4 * NUC_CAP * 8 <= SMEM_F32, "the draw's scratch fits");
 static_assert(GCAP * 4 <= HW * 4 && PCAP * 8 <= SKG * 2 && HW <= PCAP, "the aliased areas fit");
+static_assert(PCAP <= SK_TMP && GCAP * 4 <= (SK_EMASS - SK_TMP) * 8 && PCAP <= SK_EMASS - SK_TMP &&
+                  SK_EMASS + HW <= SKG / 4, "the sketch-led areas fit");
 static_assert(WCAP * 8 <= CREC * 20 && RANK_MAX * 2 <= LCAP, "the float32 work areas fit");
 
 __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
@@ -144,33 +155,45 @@ __device__ __forceinline__ float max2_value(uint32_t m2) {
     return __uint_as_float(m2);
 }
 
+// 2^(z*c - k) summed over one chunk, as a packed pair of partial sums
+template <int DT>
+__device__ __forceinline__ unsigned long long chunk_expsum2(const uint4 &x, unsigned long long c2,
+                                                            unsigned long long nk2) {
+    if (DT == ACES_BF16) {
+        const uint32_t wd[4] = {x.x, x.y, x.z, x.w};
+        unsigned long long p[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            p[q] = ex2_pair(pack2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xFFFF0000u)), c2, nk2);
+        return fadd2(fadd2(p[0], p[1]), fadd2(p[2], p[3]));
+    } else {
+        const unsigned long long p0 = ex2_pair(pack2(__uint_as_float(x.x), __uint_as_float(x.y)), c2, nk2);
+        const unsigned long long p1 = ex2_pair(pack2(__uint_as_float(x.z), __uint_as_float(x.w)), c2, nk2);
+        return fadd2(p0, p1);
+    }
+}
+
+// adds a chunk's pair s into the two accumulators (even and odd chunks)
+__device__ __forceinline__ void acc_pair(int j, unsigned long long s, unsigned long long &acc0,
+                                         unsigned long long &acc1) {
+    if (j & 1) acc1 = j == 1 ? s : fadd2(acc1, s);
+    else acc0 = j == 0 ? s : fadd2(acc0, s);
+}
+
+__device__ __forceinline__ float acc_total(unsigned long long acc0, unsigned long long acc1) {
+    float a, b;
+    unpack2(fadd2(acc0, acc1), a, b);
+    return a + b;
+}
+
 // sum over the chunks of 2^(z*c - k), two logits per instruction
 template <int DT>
 __device__ __forceinline__ float chunks_expsum(const uint4 (&w)[UC], float c, float nk) {
     const unsigned long long c2 = pack2(c, c), nk2 = pack2(nk, nk);
     unsigned long long acc0 = 0ull, acc1 = 0ull;
 #pragma unroll
-    for (int j = 0; j < UC; ++j) {
-        unsigned long long s;
-        if (DT == ACES_BF16) {
-            const uint32_t wd[4] = {w[j].x, w[j].y, w[j].z, w[j].w};
-            unsigned long long p[4];
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-                p[q] = ex2_pair(pack2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xFFFF0000u)),
-                                c2, nk2);
-            s = fadd2(fadd2(p[0], p[1]), fadd2(p[2], p[3]));
-        } else {
-            const unsigned long long p0 = ex2_pair(pack2(__uint_as_float(w[j].x), __uint_as_float(w[j].y)), c2, nk2);
-            const unsigned long long p1 = ex2_pair(pack2(__uint_as_float(w[j].z), __uint_as_float(w[j].w)), c2, nk2);
-            s = fadd2(p0, p1);
-        }
-        if (j & 1) acc1 = j == 1 ? s : fadd2(acc1, s);
-        else acc0 = j == 0 ? s : fadd2(acc0, s);
-    }
-    float a, b;
-    unpack2(fadd2(acc0, acc1), a, b);
-    return a + b;
+    for (int j = 0; j < UC; ++j) acc_pair(j, chunk_expsum2<DT>(w[j], c2, nk2), acc0, acc1);
+    return acc_total(acc0, acc1);
 }
 
 // element e of a chunk (e may be a run-time index)
@@ -306,6 +329,7 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     __shared__ int s_nrec, s_nl, s_fb, s_n, s_bsel, s_nstar, s_L, s_npay, s_ng, s_nge, s_j, s_vs, s_vk, s_nnuc;
     __shared__ float s_thlo, s_zx;
     __shared__ int s_dbins, s_xb;  // s_dbins: D in depth bins (-1: no hints yet)
+    __shared__ int s_skm;          // bfloat16: the sketch-led pass (no counting while streaming)
     __shared__ uint32_t s_mr;  // order key of the running max
     __shared__ double s_Snuc;
     __shared__ float s_inv_S;
@@ -341,9 +365,10 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     }
     // the depths published by the call's finished rows (read by warp 0 only,
     // once: they change while this row streams)
-    int hr = 0, hc0 = 0, hc1 = 0;
+    int hr = 0, hc0 = 0, hc1 = 0, hs = 0;
     if (wid == 0) {
         hr = __ldcg(&a.ws.fb_count[8]);
+        hs = __ldcg(&a.ws.fb_count[11]);
         hc0 = 2 * lane < NSB ? __ldcg(&a.ws.fb_count[WS_DEPTH + 2 * lane]) : 0;
         hc1 = 2 * lane + 1 < NSB ? __ldcg(&a.ws.fb_count[WS_DEPTH + 2 * lane + 1]) : 0;
     }
@@ -355,14 +380,18 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     // (iterations whose tiles all exist and are whole load without checks:
     // only the last iteration can hold fewer tiles, and only the row's last
     // tile can be partial)
+    // chunk u of iteration it, starting at tile `tile` (checked: bounds tested)
+    auto load_chunk = [&](int it, int u, int tile, bool checked) {
+        const int t = it * TPI + u * NWC + wid;
+        const int c = tile * TCH + lane;
+        w[u] = (!checked || (t < ntile && c < nch)) ? ldg16(row + (size_t)c * 16) : make_uint4(NI, NI, NI, NI);
+    };
     auto load = [&](int it) {
         int tile = tile0;
         const bool checked = (it + 1) * TPI > ntile || it == a.it_partial;
 #pragma unroll
         for (int u = 0; u < UC; ++u) {
-            const int t = it * TPI + u * NWC + wid;
-            const int c = tile * TCH + lane;
-            w[u] = (!checked || (t < ntile && c < nch)) ? ldg16(row + (size_t)c * 16) : make_uint4(NI, NI, NI, NI);
+            load_chunk(it, u, tile, checked);
             tile += a.pstride_w;
             if (tile >= ntile) tile -= ntile;
         }
@@ -376,7 +405,10 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     };
     // max and exp-sum of this iteration; returns mask_of(th), the iteration's
     // max in im and the maxima of chunks 0..3 and 4..7 in g0, g1
-    auto math = [&](float th, float &im, float &g0, float &g1) -> uint32_t {
+    // the iteration's maxima and the reference k_t raised to them; returns
+    // mask_of(th), the iteration's max in im and the maxima of chunks 0..3
+    // and 4..7 in g0, g1
+    auto head = [&](float th, float &im, float &g0, float &g1) -> uint32_t {
         uint32_t hb = 0u;
         g0 = -INFINITY;
         g1 = -INFINITY;
@@ -397,11 +429,18 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
             e_t *= sc;
             k_t = nk;
         }
-        const float gs = chunks_expsum<DT>(w, a.c, -k_t);
+        return hb;
+    };
+    auto add_sum = [&](float gs) {
         const float t = s_t + gs;  // Neumaier
         if (fabsf(s_t) >= fabsf(gs)) e_t += (s_t - t) + gs;
         else e_t += (gs - t) + s_t;
         s_t = t;
+    };
+    // max and exp-sum of this iteration (head, then the sum)
+    auto math = [&](float th, float &im, float &g0, float &g1) -> uint32_t {
+        const uint32_t hb = head(th, im, g0, g1);
+        add_sum(chunks_expsum<DT>(w, a.c, -k_t));
         return hb;
     };
     // the running max of the CTA (a lower bound of the row max at any time)
@@ -430,7 +469,11 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         const int hb = (float)(inc - hc1) >= need ? 2 * lane : ((float)inc >= need ? 2 * lane + 1 : NSB);
         const unsigned bal = __ballot_sync(0xffffffffu, hb < NSB);
         const int hq = bal ? __shfl_sync(0xffffffffu, hb, __ffs(bal) - 1) : NSB - 1;
-        if (lane == 0) s_dbins = hr >= HINT_MIN ? min(hq + HINT_MARGIN, NSB - 1) + 1 : -1;
+        if (lane == 0) {
+            s_dbins = hr >= HINT_MIN ? min(hq + HINT_MARGIN, NSB - 1) + 1 : -1;
+            // the sketch-led pass when nearly every finished row was short
+            s_skm = BF && hr >= HINT_MIN && (long long)hs * SHORT_DEN >= (long long)hr * SHORT_NUM;
+        }
     }
     publish_max(im);
     __syncthreads();
@@ -449,6 +492,7 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     float m = -INFINITY, kref = -1e30f;
     double S = 0.0;
     float v_need = 0.0f;  // the crossing (top_p = 1: the payload's end), for the hints
+    bool short_row = false;  // (bfloat16) few ids reach the crossing: published for later rows' pass
 
     // reduces the row max, the reference and the exp-sum (fp32 two-sum tree,
     // fp64 in warp 0); true when the row is not a distribution (handled)
@@ -518,7 +562,8 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         // chunks of 2^ish iterations).
         uint32_t thb0 = 1u;
         bool count_on = false;
-        if (have && m1 > 0.0f) {
+        const bool skm = s_skm != 0;
+        if (have && m1 > 0.0f && !skm) {
             const float t = m1 - D;
             int lo = t > 0.0f ? (int)__bfloat16_as_ushort(__float2bfloat16_rd(t)) : 1;
             lo = max(lo, (int)(__float_as_uint(m1) >> 16) + HEADROOM - (HW - 1));
@@ -537,28 +582,21 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         // (the counts' shared-memory address, offset so that a value's bit
         // pattern times 4 indexes its counter)
         const uint32_t hbase = (uint32_t)__cvta_generic_to_shared(hist) - thb0 * 4u;
-        auto count_hits = [&](uint32_t hb, uint32_t thb) {
-            // chunk positions where some lane of the warp reaches thb (the
-            // branches are warp-uniform; every lane checks every element)
-            const uint32_t any = __reduce_or_sync(0xffffffffu, hb);
-            if (any == 0u) return;
+        // counts the ids of chunk u that reach thb (every lane checks every
+        // element: the callers' branches are warp-uniform)
+        auto count_chunk = [&](int u, uint32_t thb) {
             const uint32_t span = thb0 + HW - thb;
+            const uint32_t wd[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
 #pragma unroll
-            for (int u = 0; u < UC; ++u) {
-                if ((any >> u) & 1u) {
-                    const uint32_t wd[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint32_t lo = wd[q] & 0xFFFFu, hi = wd[q] >> 16;
+            for (int q = 0; q < 4; ++q) {
+                const uint32_t lo = wd[q] & 0xFFFFu, hi = wd[q] >> 16;
 #ifdef ACES_CHECKED
-                        if (lo - thb < span && ACES_IN(lo - thb0, HW)) atomicAdd(&hist[lo - thb0], 1u);
-                        if (hi - thb < span && ACES_IN(hi - thb0, HW)) atomicAdd(&hist[hi - thb0], 1u);
+                if (lo - thb < span && ACES_IN(lo - thb0, HW)) atomicAdd(&hist[lo - thb0], 1u);
+                if (hi - thb < span && ACES_IN(hi - thb0, HW)) atomicAdd(&hist[hi - thb0], 1u);
 #else
-                        red_inc_lt(hbase + lo * 4u, lo - thb, span);
-                        red_inc_lt(hbase + hi * 4u, hi - thb, span);
+                red_inc_lt(hbase + lo * 4u, lo - thb, span);
+                red_inc_lt(hbase + hi * 4u, hi - thb, span);
 #endif
-                    }
-                }
             }
         };
         const int gpi = a.sk_gpi, ish = a.sk_ish;
@@ -593,7 +631,13 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
                     hb = math(thf, im, g0, g1);
                     publish_max(im);
                 }
-                if (count_on) count_hits(hb, thb);
+                if (count_on) {
+                    // chunk positions where some lane of the warp reaches thb
+                    const uint32_t any = __reduce_or_sync(0xffffffffu, hb);
+#pragma unroll
+                    for (int u = 0; u < UC; ++u)
+                        if ((any >> u) & 1u) count_chunk(u, thb);
+                }
                 sketch_put(it);
             }
         }
@@ -775,6 +819,7 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
                 if (ACES_IN(slot, SKG) && sk[slot] >= key) hm |= 1ull << i;
             }
             int at = warp_place(__popcll(hm), &s_ng);
+            __syncthreads();  // (gl may overlap slots of the sketch read above)
             while (hm) {
                 const int i = __ffsll((long long)hm) - 1;
                 hm &= hm - 1ull;
@@ -839,11 +884,120 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         auto put_pay = [&](int at, uint32_t bits, uint32_t id) {
             if (at < PCAP && ACES_IN(at, PCAP)) pay[at] = order_val(fkey(__uint_as_float(bits << 16)), id);
         };
+        // ---- sketch-led pass (rows of a call whose finished rows were
+        // short; nothing was counted while streaming).  The group maxima
+        // bound the mass above each value from below (one id per group), so
+        // the value vl where that bound reaches top_p * S (top_p = 1: where
+        // k groups are reached) lies at or below the crossing (the payload's
+        // end); the groups reaching vl are read back, their ids >= vl counted
+        // and kept, and the scan of those exact counts follows.  Returns 0
+        // (pay holds the ids >= the scan's vr), 1 when the second counting
+        // pass is needed, 2 when the row goes to the general kernel ----
+        auto sketch_led = [&]() -> int {
+            thb0 = km > (uint32_t)(HW - 1) ? km - (uint32_t)(HW - 1) : 1u;
+            for (int slot = tid; slot < ng_all; slot += NTC) {  // (hist is clear)
+                const uint32_t key = ACES_IN(slot, SKG) ? (uint32_t)sk[slot] : 0u;
+                const uint32_t idx = key - 0x8000u - thb0;
+                if (key >= 0x8000u + thb0 && idx < (uint32_t)HW) atomicAdd(&hist[idx], 1u);
+            }
+            __syncthreads();
+            if (wid == 0) {
+                const unsigned long long tg =
+                    all_in ? 0ull : (unsigned long long)ceil((double)a.top_p * S * (double)FX_SCALE);
+                const int top = (int)(km - thb0);
+                const int per = (top + 32) >> 5;
+                const int b0 = top - lane * per;  // this lane's values: b0, b0 - 1, ... (>= 0)
+                unsigned long long lm = 0ull, lc = 0ull;
+                for (int i = 0; i < per; ++i) {
+                    const int idx = b0 - i;
+                    if (idx < 0) break;
+                    const uint32_t cn = hist[idx];
+                    if (cn) {
+                        lm += (unsigned long long)cn * vmass(idx);
+                        lc += cn;
+                    }
+                }
+                unsigned long long incm = lm, incc = lc;
+                for (int o = 1; o < 32; o <<= 1) {
+                    const unsigned long long tm = __shfl_up_sync(0xffffffffu, incm, o);
+                    const unsigned long long tc = __shfl_up_sync(0xffffffffu, incc, o);
+                    if (lane >= o) {
+                        incm += tm;
+                        incc += tc;
+                    }
+                }
+                int vl = -1;
+                const bool mine = all_in ? (incc - lc < (unsigned long long)a.k && incc >= (unsigned long long)a.k)
+                                         : (incm - lm < tg && incm >= tg);
+                if (mine) {
+                    unsigned long long cm = incm - lm, cc = incc - lc;
+                    for (int i = 0; i < per; ++i) {
+                        const int idx = b0 - i;
+                        if (idx < 0) break;
+                        const uint32_t cn = hist[idx];
+                        if (!cn) continue;
+                        cm += (unsigned long long)cn * vmass(idx);
+                        cc += cn;
+                        if (all_in ? cc >= (unsigned long long)a.k : cm >= tg) {
+                            vl = idx;
+                            break;
+                        }
+                    }
+                }
+                const unsigned bal = __ballot_sync(0xffffffffu, vl >= 0);
+                vl = bal ? __shfl_sync(0xffffffffu, vl, __ffs(bal) - 1) : -1;
+                if (lane == 0) s_bsel = vl;
+            }
+            __syncthreads();
+            const int vl = s_bsel;
+            if (vl < 0) return 1;
+            const uint32_t vlb = thb0 + (uint32_t)vl;
+            uint32_t *gls = reinterpret_cast<uint32_t *>(reinterpret_cast<unsigned long long *>(sk) + SK_TMP);
+            const int ng = compact(0x8000u + vlb, gls);
+            if (ng > GCAP) return 1;
+            for (int i = tid; i < HW; i += NTC) hist[i] = 0u;
+            if (tid == 0) s_npay = 0;
+            __syncthreads();
+            reread(gls, ng, vlb, &s_npay, [&](int at, uint32_t bits, uint32_t id) {
+                const uint32_t idx = bits - thb0;
+                if (idx < (uint32_t)HW) atomicAdd(&hist[idx], 1u);
+                if (at < PCAP && ACES_IN(at, PCAP)) pay[at] = order_val(fkey(__uint_as_float(bits << 16)), id);
+            });
+            const int nall = s_npay;
+            if (nall > PCAP) return 1;
+            emass = reinterpret_cast<unsigned long long *>(sk) + SK_EMASS;
+            const int f = scan(vlb);
+            if (f != 0) return f;
+            // keep in pay the ids >= the scan's vr
+            if (s_vk >= 0) {
+                const uint32_t kr = fkey(val16(0x8000u + thb0 + (uint32_t)s_vk));
+                unsigned long long *tmp = reinterpret_cast<unsigned long long *>(sk) + SK_TMP;
+                for (int i0 = 0; i0 < nall; i0 += NTC) {  // warp-uniform rounds
+                    const int i = i0 + tid;
+                    const unsigned long long o = i < nall ? pay[i] : 0ull;
+                    const bool keep = i < nall && (uint32_t)(o >> 32) >= kr;
+                    const int at = warp_place(keep ? 1 : 0, &s_npay);
+                    if (keep && ACES_IN(at, PCAP)) tmp[at] = o;
+                }
+                __syncthreads();
+                const int nk = s_npay;
+                for (int i = tid; i < nk; i += NTC)
+                    if (ACES_IN(i, PCAP)) pay[i] = tmp[i];
+                __syncthreads();
+            }
+            return 0;
+        };
         int fb = 1;
-        if (count_on && km < thb0 + HW) {
+        bool pay_ready = false;  // (sketch-led) pay holds the ids >= vr
+        if (skm) {
+            fb = sketch_led();
+            pay_ready = fb == 0;
+            if (tid == 0 && fb == 0) atomicAdd(&a.ws.fb_count[12], 1);
+        } else if (count_on && km < thb0 + HW) {
             fb = scan(lim_of(m));
         }
         if (fb == 1) {
+            emass = pay;
             // the crossing (or the row max) lies outside the counted values:
             // a second pass counts the row again, from the row max down as far
             // as the window reaches
@@ -883,7 +1037,7 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         if (vr >= 0) {
             // ---- the ids at or above value vr, then ordered ----
             const uint32_t vrb = thb0 + (uint32_t)vr;  // its bit pattern
-            {
+            if (!pay_ready) {
                 const int ng = compact(0x8000u + vrb, glist);
                 if (ng > GCAP) {
                     if (tid == 0) fallback_row(a, r, m, kref, S);
@@ -963,6 +1117,7 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
             }
         }
         v_need = all_in ? (L > 0 ? order_value(ord[L - 1]) : m) : val16(0x8000u + vsb);
+        short_row = all_in ? a.k <= SHORT_IDS : (n_nuc >= 0 && n_nuc <= SHORT_IDS);
         if (tid == 0) atomicAdd(&a.ws.fb_count[2], 1);
     } else {
         // ================= float32: list mode =================
@@ -1302,6 +1457,7 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         if (ACES_IN(dx, NSB)) atomicAdd(&a.ws.fb_count[WS_DEPTH + dx], 1);
         atomicAdd(&a.ws.fb_count[8], 1);
         if (hinted) atomicAdd(&a.ws.fb_count[9], 1);
+        if (short_row) atomicAdd(&a.ws.fb_count[11], 1);
     }
     const float inv_S = s_inv_S;
     for (int j = tid; j < a.k; j += NTC) {

@@ -26,7 +26,8 @@ pytestmark = pytest.mark.gpu
 
 torch = pytest.importorskip("torch")
 
-FALLBACK, TIMEOUTS, VALUE_MODE, BITONIC, RADIX, LAZY, GEN_VALHIST, TIE_RANK, PUBLISHED, HINTED, RECOUNT = range(11)
+(FALLBACK, TIMEOUTS, VALUE_MODE, BITONIC, RADIX, LAZY, GEN_VALHIST, TIE_RANK, PUBLISHED, HINTED, RECOUNT, SHORT,
+ SKETCH_LED) = range(13)
 
 
 @pytest.fixture(scope="module")
@@ -279,6 +280,36 @@ def test_later_rows_take_their_depth_from_finished_rows(A, orc, dtype):
     # (float32 rows whose capture overflows the 1536 recorded chunks go to
     # the exact general kernel)
     assert counters[HINTED] >= 200 and counters[FALLBACK] <= (8 if dtype == "bf16" else 200), counters
+    assert res["checked_seqs"] >= 32
+
+
+def test_short_rows_lead_later_rows_to_the_sketch(A, orc):
+    # 1088 rows shaped like the 256000-id workload (T = 0.6, top_p = 0.8,
+    # k = 128: nuclei of tens of ids).  Once 32 rows have finished, all of
+    # them short, later rows stream without counting and read back only the
+    # sketch groups that can hold the nucleus.
+    w = gen.make_workload(64, 16, 256000, "bf16", sigma=3.0, rho=0.9, T=0.6, top_p=0.8, k=128, seed=57)
+    inp = gen.generate(w)
+    counters, res = _run(A, orc, w, inp["z"], inp=dict(inp))
+    assert counters[FALLBACK] == 0 and counters[SHORT] >= 200 and counters[SKETCH_LED] >= 200, counters
+    assert res["checked_seqs"] >= 32
+
+
+def test_sketch_led_row_with_a_long_nucleus_counts_again(A, orc):
+    # The first 800 rows have four dominant ids (short nuclei), the last
+    # 288 flat logits (nuclei of most of the row).  Rows that start after
+    # the short ones finished take the sketch-led pass; for the flat ones
+    # the groups it marks do not hold the crossing, and the row is counted
+    # in a second pass instead.
+    B, K, V = 64, 16, 32768
+    w = gen.make_workload(B, K, V, "bf16", T=1.0, top_p=0.9, k=16, seed=58)
+    rng = np.random.default_rng(58)
+    rows = B * (K + 1)
+    z = rng.uniform(0.0, 1.0, size=(rows, V)).astype(np.float32)
+    for r in range(800):
+        z[r, rng.choice(V, 4, replace=False)] = 12.0 + rng.uniform(0.0, 0.5, 4)
+    counters, res = _run(A, orc, w, _bf16(z.reshape(B, K + 1, V)))
+    assert counters[FALLBACK] == 0 and counters[SKETCH_LED] >= 100 and counters[RECOUNT] >= 1, counters
     assert res["checked_seqs"] >= 32
 
 
