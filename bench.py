@@ -372,7 +372,7 @@ def per_config(A, torch, dev, stream, peak, peak_kind, have=None, cpu=True):
             e1.record(stream)
         torch.cuda.synchronize()
         vms = statistics.median(e0.elapsed_time(e1) for e0, e1 in ev)
-        paths = dict(zip(PATHS, wsb[:64].view(torch.int32).cpu().numpy().tolist()))
+        paths = dict(zip(PATHS, wsb[A.COUNTERS_OFFSET:A.COUNTERS_OFFSET + 64].view(torch.int32).cpu().numpy().tolist()))
         paths.pop("timeouts")
         vb = verify_bytes(B, K, V, k, zsize, resid_q_count(out, K, k))
         for _ in range(3):
@@ -525,7 +525,7 @@ def main():
     al = out["accept_len"].cpu().numpy()
     n_rej = int((al < K).sum())
     n_resid_q = resid_q_count(out, K, k)
-    paths = dict(zip(PATHS, wsb[:64].view(torch.int32).cpu().numpy().tolist()))
+    paths = dict(zip(PATHS, wsb[A.COUNTERS_OFFSET:A.COUNTERS_OFFSET + 64].view(torch.int32).cpu().numpy().tolist()))
     paths.pop("timeouts")
     peak, peak_kind = measured_peak()
     vb = verify_bytes(B, K, V, k, zsize, n_resid_q)

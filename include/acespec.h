@@ -144,7 +144,7 @@ aces_status aces_verify(const void *target_logits, aces_dtype dt, const float *d
  * library, kept on every GPU that loads the library until the process exits.
  * This call allocates nothing.
  *   - Size limit: returns ACES_ERR_UNSUPPORTED (nothing launched) when
- *     B > 876 at K = 16, B > 1196 at K = 8, B > 1464 at K = 4 (the limit
+ *     B > 876 at K = 16, B > 1196 at K = 8, B > 1463 at K = 4 (the limit
  *     does not depend on V or k).  The scratch keeps nucleus lists only for
  *     B <= 14 at K = 16 (27 at K = 8, 49 at K = 4); without them the
  *     residual draw scans its whole row.  The results are the same either

@@ -22,7 +22,7 @@ import threading
 import torch
 
 __all__ = ["load", "use_checked", "checked_violation", "lib_path", "workspace_bytes", "verify", "sparsify", "cache_build", "cache_lookup",
-           "ROW_NONFINITE", "ROW_BAD_Q", "AcespecError"]
+           "ROW_NONFINITE", "ROW_BAD_Q", "COUNTERS_OFFSET", "AcespecError"]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "libacespec.so")
@@ -30,6 +30,10 @@ _LIB_CHECKED = os.path.join(_HERE, "libacespec_checked.so")
 _lock = threading.Lock()
 _lib = None          # the library every function below calls
 _libs = {}           # loaded libraries by path
+
+# byte offset of the 16 path counters in a workspace (int32; after the hints
+# a call leaves for the next one)
+COUNTERS_OFFSET = 256
 
 ROW_NONFINITE = 1
 ROW_BAD_Q = 2

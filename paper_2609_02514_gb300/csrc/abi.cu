@@ -137,6 +137,9 @@ aces_status aces::verify_impl(const void *target_logits, aces_dtype dt, const fl
     r.B = B;
     r.K = K;
     r.V = V;
+    r.T = T;
+    r.top_p = top_p;
+    r.k = k;
     r.ws = a.ws;
     r.accept_len = accept_len;
     r.out_token = out_token;

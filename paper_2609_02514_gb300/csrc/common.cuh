@@ -360,10 +360,16 @@ struct SegSum {
 constexpr int NSEG_MAX = 16;
 constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual step
 
-constexpr int WS_COUNTERS = 256;      // bytes of path counters and depth hints at the start of the workspace
+constexpr int WS_CARRY = 256;         // bytes of the hints carried from the previous call, at the start
+constexpr int WS_COUNTERS = 256;      // bytes of path counters and depth hints, after them
 constexpr int WS_DEPTH = 16;          // first of the 40 depth counters of the row kernel's hints (int index)
+constexpr int CARRY_MAGIC = 0x41434531;  // marks a written carry area
 // Workspace layout (all offsets 16-byte aligned)
 struct Workspace {
+    int *carry;                // [64] never cleared: the previous call's hints (written by the resolve
+                               //       step): [0] CARRY_MAGIC, [1] T bits, [2] top_p bits, [3] k, [4] V,
+                               //       [5] dtype, [6] rows that published a depth, [7] short rows,
+                               //       [16..55] how many rows needed each depth
     int *fb_count;             // [64] path counters and depth hints, cleared by every call: [0] rows handed to the
                                //       general kernel, [1] reserved (no kernel waits on another),
                                //       [2] bfloat16 rows finished from their value counts, [3] rows
@@ -389,7 +395,7 @@ __host__ __device__ inline size_t align16(size_t x) { return (x + 15) & ~(size_t
 // rows = B*(K+1) target rows; nseq = B sequences with K draft positions (K = 0: sparsify);
 // lists: keep every row's nucleus (up to NUC_CAP ids) for the residual step
 __host__ __device__ inline size_t ws_bytes(int rows, int nseq, int K, bool lists) {
-    size_t b = WS_COUNTERS + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
+    size_t b = WS_CARRY + WS_COUNTERS + align16((size_t)rows * sizeof(RowStat)) + align16((size_t)nseq * K * 4) +
                align16((size_t)rows * 4);
     if (K > 0) {
         b += 2 * align16((size_t)nseq * 4) + align16((size_t)nseq * NSEG_MAX * sizeof(SegSum));
@@ -407,6 +413,8 @@ __host__ __device__ inline size_t ws_clear_bytes(int nseq, int K) {
 __host__ __device__ inline Workspace ws_carve(void *base, int rows, int nseq, int K, bool lists) {
     char *p = (char *)base;
     Workspace w;
+    w.carry = (int *)p;
+    p += WS_CARRY;
     w.fb_count = (int *)p;
     p += WS_COUNTERS;
     w.seqcnt = nullptr;
@@ -472,6 +480,8 @@ struct ResolveArgs {
     const float *q;
     const float *u;
     int B, K, V;
+    float T, top_p;  // (with k: the key of the hints carried to the next call)
+    int k;
     Workspace ws;
     int32_t *accept_len;
     int32_t *out_token;

@@ -189,6 +189,22 @@ template <int DT, bool VEC>
 __global__ void __launch_bounds__(NTS, 2) k_resolve_seg(ResolveArgs a, int nseg, int seglen, int tps, int tpw) {
     pdl_wait();  // the row kernels are complete
     const int lane = threadIdx.x & 31;
+    if (blockIdx.x == 0 && threadIdx.x < WS_COUNTERS / 4) {
+        // the hints of this call's rows, for the first rows of the next call
+        // with the same shape (the row kernels read them only when fewer
+        // than their minimum of this call's rows have finished)
+        const int i = threadIdx.x;
+        int v = i >= WS_DEPTH ? __ldcg(&a.ws.fb_count[i]) : 0;
+        if (i == 0) v = CARRY_MAGIC;
+        if (i == 1) v = __float_as_int(a.T);
+        if (i == 2) v = __float_as_int(a.top_p);
+        if (i == 3) v = a.k;
+        if (i == 4) v = a.V;
+        if (i == 5) v = DT;
+        if (i == 6) v = __ldcg(&a.ws.fb_count[8]);
+        if (i == 7) v = __ldcg(&a.ws.fb_count[11]);
+        a.ws.carry[i] = v;
+    }
     const long long gw = (long long)blockIdx.x * (NTS / 32) + (threadIdx.x >> 5);
     const long long ntask = (long long)a.B * tps;
     const long long t_lo = gw * tpw;

@@ -52,7 +52,7 @@ def _run(A, orc, w, z, exact=False, inp=None):
     g = A.verify(zt, q, xt, u, w.T, w.top_p, w.k, workspace=ws, exact=exact)
     torch.cuda.synchronize()
     g = {key: v.cpu().numpy() for key, v in g.items()}
-    counters = ws[:64].view(torch.int32).cpu().numpy().tolist()
+    counters = ws[A.COUNTERS_OFFSET:A.COUNTERS_OFFSET + 64].view(torch.int32).cpu().numpy().tolist()
     o = orc.verify(z, inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
     res = parity.compare_verify(inp, g, o, w.top_p, z.dtype == np.uint16, w.k)
     return counters, res
