@@ -460,7 +460,7 @@ def main():
     out = A.verify(d["z"], d["q"], d["xt"], d["u"], w.T, w.top_p, k)
     cache = A.cache_build(d["q"], d["xt"], w.F)
     slot = A.cache_lookup(cache["branch_tok"], w.F, out["accept_len"], out["out_token"])
-    wsb = torch.empty(A.workspace_bytes(B, K, V, k), dtype=torch.uint8, device=dev)
+    wsb = torch.zeros(A.workspace_bytes(B, K, V, k), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
     stream = torch.cuda.current_stream(dev)
 
@@ -650,7 +650,7 @@ def main():
                 continue
             sub = {key: d[key][:bs] for key in ("z", "q", "xt", "u")}
             o2 = A.verify(sub["z"], sub["q"], sub["xt"], sub["u"], w.T, w.top_p, k)
-            ws2 = torch.empty(A.workspace_bytes(bs, K, V, k), dtype=torch.uint8, device=dev)
+            ws2 = torch.zeros(A.workspace_bytes(bs, K, V, k), dtype=torch.uint8, device=dev)
             for _ in range(3):
                 A.verify(sub["z"], sub["q"], sub["xt"], sub["u"], w.T, w.top_p, k, out=o2, workspace=ws2)
             e0 = torch.cuda.Event(enable_timing=True)

@@ -88,7 +88,13 @@ typedef struct CUstream_st *aces_stream_t;
  * draw when it has at most 512 ids), under 100 bytes per row for
  * aces_sparsify.  The caller allocates it, passes it to the call and must
  * not use it while the call's work is in flight; it needs no
- * initialisation.  Returns 0 for invalid sizes.
+ * initialisation.  Its first 256 bytes keep, from one aces_verify call to
+ * the next on the same workspace, statistics of the rows (how deep below
+ * their max their nucleus ended, how many were short) that let the row
+ * kernel pick its pass before enough of the new call's rows have finished;
+ * they choose a pass only, never a result, so any content there (a fresh
+ * allocation, another shape's call) gives the same outputs.  Returns 0 for
+ * invalid sizes.
  */
 size_t aces_workspace_bytes(int B, int K, int V, int k);
 

@@ -50,6 +50,11 @@ aces_status run_rows(RowArgs &a, aces_dtype dt, bool exact, cudaStream_t s) {
     const int nseq = a.K > 0 ? a.rows / (a.K + 1) : a.rows;
     if (cudaMemsetAsync(a.ws.fb_count, 0, ws_clear_bytes(nseq, a.K), s) != cudaSuccess) return ACES_ERR_CUDA;
     const int grid = a.rows < 2 * nsm ? a.rows : 2 * nsm;
+    a.nsm = nsm;
+    // With many waves of rows the four CTAs an SM starts with would reach
+    // their epilogues (when few loads are in flight) together, wave after
+    // wave: their starts are spread over about a quarter of a row's time.
+    a.stagger_ns = a.rows >= 16 * nsm ? STAGGER_NS : 0;
     if (vec) {
         rows_cap_layout(a, dt);
         a.force_fb = exact ? 1 : 0;

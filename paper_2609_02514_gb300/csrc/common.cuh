@@ -112,6 +112,11 @@ __device__ __forceinline__ float order_value(unsigned long long o) {
 // row kernel never triggers early: general-kernel CTAs placed on the first
 // SMs its last wave frees would crowd there and unbalance that persistent
 // grid.  Without the launch attribute both calls are no-ops.
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
@@ -358,6 +363,7 @@ struct SegSum {
     int nt;                 // ids of a lazy cut's value
 };
 constexpr int NSEG_MAX = 16;
+constexpr int STAGGER_NS = 10000;  // row kernel: first-wave start spread per CTA of an SM
 constexpr int NUC_CAP = 512;  // nucleus entries kept per row for the residual step
 
 constexpr int WS_CARRY = 256;         // bytes of the hints carried from the previous call, at the start
@@ -472,6 +478,8 @@ struct RowArgs {
     int sk_gpi, sk_ish;    // bfloat16 sketch: groups per thread and iteration (2: 4 chunks each; 1: 8
                            // chunks of 2^sk_ish iterations)
     int force_fb;          // hand every row to the general kernel (the library's exact reference path)
+    int nsm;               // SMs of the device
+    int stagger_ns;        // start of the first-wave CTAs of an SM spread by this (0: none)
 };
 
 // Arguments of the sequence kernel.

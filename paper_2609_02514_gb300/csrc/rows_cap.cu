@@ -338,6 +338,14 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
 
     const int r = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    if (a.stagger_ns > 0 && r < 4 * a.nsm) {
+        // the j-th CTA an SM starts with (blocks are placed on the SMs in
+        // turn) waits j times stagger_ns on the global timer (bounded: at
+        // most 3 x stagger_ns)
+        const unsigned long long wait = (unsigned long long)(r / a.nsm) * (unsigned long long)a.stagger_ns;
+        const unsigned long long t0 = globaltimer_ns();
+        for (int i = 0; i < 1000 && globaltimer_ns() - t0 < wait; ++i) __nanosleep(1000);
+    }
     const char *row = reinterpret_cast<const char *>(a.logits) + (size_t)r * a.V * E::SIZE;
     const int nch = a.V / EPC, ntile = a.ntile;
     const int nit = (ntile + TPI - 1) / TPI;
