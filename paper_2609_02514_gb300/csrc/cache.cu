@@ -76,9 +76,21 @@ __global__ void __launch_bounds__(NTC, 4) k_cache_build(CacheArgs a) {
                     thr = t > 1u ? t : 1u;
                 }
             };
+            // Fd <= TOPL: a lane's Fd-th entry bounds the Fd largest of the
+            // row from below (that lane alone holds Fd values at or above
+            // it), so the warp's largest such entry raises every lane's
+            // threshold; refreshed once per round of loads (the filter then
+            // drops what no list could keep, and insertions stay rare)
             if (VEC) {
                 const int nch = a.V >> 2;
                 for (int c0 = tid; c0 < nch; c0 += NTC * CLD) {
+                    if (TOPL == 8 && c0 != tid && Fd <= TOPL) {  // (warp-uniform; the short lists filter enough)
+                        unsigned long long e = 0ull;
+#pragma unroll
+                        for (int i = 0; i < TOPL; ++i) e = i == Fd - 1 ? Lst[i] : e;
+                        const uint32_t wb = __reduce_max_sync(0xffffffffu, (uint32_t)(e >> 32) & 0x7FFFFFFFu);
+                        thr = wb > thr ? wb : thr;
+                    }
                     uint4 w[CLD];
 #pragma unroll
                     for (int u = 0; u < CLD; ++u) {
