@@ -97,15 +97,37 @@ __global__ void __launch_bounds__(NTC, 4) k_cache_build(CacheArgs a) {
                         const int cc = c0 + u * NTC;
                         w[u] = cc < nch ? ldg16(qr + (size_t)cc * 4) : make_uint4(0u, 0u, 0u, 0u);
                     }
+                    if (TOPL == 8) {
+                        // the values reaching thr as bits of one mask, then
+                        // one insertion site in a loop over them (unrolled
+                        // sites of the eight-entry insertion overflow the
+                        // instruction cache)
+                        uint32_t mk = 0u;
 #pragma unroll
-                    for (int u = 0; u < CLD; ++u) {
-                        // one test per four values: the largest raw bits
-                        if (max(max(w[u].x, w[u].y), max(w[u].z, w[u].w)) >= thr) {
-                            const int x0 = (c0 + u * NTC) * 4;
-                            if (w[u].x >= thr) consider(__uint_as_float(w[u].x), x0);
-                            if (w[u].y >= thr) consider(__uint_as_float(w[u].y), x0 + 1);
-                            if (w[u].z >= thr) consider(__uint_as_float(w[u].z), x0 + 2);
-                            if (w[u].w >= thr) consider(__uint_as_float(w[u].w), x0 + 3);
+                        for (int u = 0; u < CLD; ++u)
+                            mk |= ((uint32_t)(w[u].x >= thr) | (uint32_t)(w[u].y >= thr) << 1 |
+                                   (uint32_t)(w[u].z >= thr) << 2 | (uint32_t)(w[u].w >= thr) << 3) << (4 * u);
+                        while (mk) {
+                            const int bit = __ffs(mk) - 1;
+                            mk &= mk - 1u;
+                            const int u = bit >> 2, j = bit & 3;
+                            uint4 x = w[0];
+#pragma unroll
+                            for (int k = 1; k < CLD; ++k) x = u == k ? w[k] : x;
+                            const uint32_t v = j == 0 ? x.x : j == 1 ? x.y : j == 2 ? x.z : x.w;
+                            consider(__uint_as_float(v), (c0 + u * NTC) * 4 + j);
+                        }
+                    } else {
+#pragma unroll
+                        for (int u = 0; u < CLD; ++u) {
+                            // one test per four values: the largest raw bits
+                            if (max(max(w[u].x, w[u].y), max(w[u].z, w[u].w)) >= thr) {
+                                const int x0 = (c0 + u * NTC) * 4;
+                                if (w[u].x >= thr) consider(__uint_as_float(w[u].x), x0);
+                                if (w[u].y >= thr) consider(__uint_as_float(w[u].y), x0 + 1);
+                                if (w[u].z >= thr) consider(__uint_as_float(w[u].z), x0 + 2);
+                                if (w[u].w >= thr) consider(__uint_as_float(w[u].w), x0 + 3);
+                            }
                         }
                     }
                 }
