@@ -379,9 +379,11 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         hs = __ldcg(&a.ws.fb_count[11]);
         hc0 = 2 * lane < NSB ? __ldcg(&a.ws.fb_count[WS_DEPTH + 2 * lane]) : 0;
         hc1 = 2 * lane + 1 < NSB ? __ldcg(&a.ws.fb_count[WS_DEPTH + 2 * lane + 1]) : 0;
-        if (hr < HINT_MIN) {
+        if (BF && hr < HINT_MIN) {
             // too few yet: those the previous call on this workspace carried,
-            // when it had the same T, top_p, k, V and logit type
+            // when it had the same T, top_p, k, V and logit type (bfloat16
+            // rows: a float32 row's capture from its own sample overflows
+            // less often than from the carried depth)
             const int *cy = a.ws.carry;
             const bool same = __ldcg(cy) == CARRY_MAGIC && __ldcg(cy + 1) == __float_as_int(a.T) &&
                               __ldcg(cy + 2) == __float_as_int(a.top_p) && __ldcg(cy + 3) == a.k &&
