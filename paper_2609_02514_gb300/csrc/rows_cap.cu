@@ -1350,14 +1350,55 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
                 }
             }
         } else {
+            // more: bin by bin (the bins of T/8 below m order the values), and
+            // inside a bin by direct ranking among its own ids
             if (tid == 0) atomicAdd(&a.ws.fb_count[3], 1);
-            ord = list;
-            efx = work;
-            const int np = next_pow2(n);
-            for (int i = tid; i < np; i += NTC)
-                if (ACES_IN(i, LCAP)) ord[i] = i < n ? cv[i] : 0ull;
+            auto bin_of = [&](unsigned long long o) -> int {
+                const float d = (m - order_value(o)) * a.inv_w;
+                return d < (float)(NBIN - 1) ? (int)d : NBIN - 1;
+            };
+            if (wid == 0) {  // bcnt[b] <- the first place of bin b (bins 0..bsel hold the candidates)
+                constexpr int PER = NBIN / 32;
+                uint32_t c[PER], loc = 0u;
+#pragma unroll
+                for (int j = 0; j < PER; ++j) {
+                    const int bn = lane * PER + j;
+                    c[j] = bn <= bsel ? bcnt[bn] : 0u;
+                    loc += c[j];
+                }
+                uint32_t inc = loc;
+                for (int o = 1; o < 32; o <<= 1) {
+                    const uint32_t t = __shfl_up_sync(0xffffffffu, inc, o);
+                    if (lane >= o) inc += t;
+                }
+                uint32_t run = inc - loc;
+#pragma unroll
+                for (int j = 0; j < PER; ++j) {
+                    bcnt[lane * PER + j] = run;
+                    run += c[j];
+                }
+            }
             __syncthreads();
-            bitonic_sort_desc(ord, np);
+            unsigned long long *binned = list;
+            for (int i = tid; i < n; i += NTC) {
+                const unsigned long long o = ACES_IN(i, WCAP) ? cv[i] : 0ull;
+                const int bn = bin_of(o);
+                const uint32_t at = ACES_IN(bn, NBIN) ? atomicAdd(&bcnt[bn], 1u) : 0u;
+                if (ACES_IN(at, LCAP)) binned[at] = o;
+            }
+            __syncthreads();  // (bcnt[b] is now the end of bin b)
+            ord = work;
+            for (int i = tid; i < n; i += NTC) {
+                const unsigned long long o = ACES_IN(i, LCAP) ? binned[i] : 0ull;
+                const int bn = bin_of(o);
+                const int st = bn > 0 && ACES_IN(bn - 1, NBIN) ? (int)bcnt[bn - 1] : 0;
+                const int en = ACES_IN(bn, NBIN) ? (int)bcnt[bn] : 0;
+                int rank = 0;
+                for (int j = st; j < en; ++j) rank += (ACES_IN(j, LCAP) ? binned[j] : 0ull) > o;
+                if (ACES_IN(st + rank, WCAP)) ord[st + rank] = o;
+            }
+            __syncthreads();
+            efx = list;
             for (int i = tid; i < n; i += NTC)
                 if (ACES_IN(i, WCAP)) efx[i] = id_fx(order_value(ord[i]), a.c, kref);
         }

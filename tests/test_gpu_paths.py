@@ -295,6 +295,48 @@ def test_short_rows_lead_later_rows_to_the_sketch(A, orc):
     assert res["checked_seqs"] >= 32
 
 
+def _verify_ws(A, w, inp, ws):
+    zt = torch.from_numpy(inp["z"].view(np.int16)).cuda().view(torch.bfloat16)
+    q, xt, u = (torch.from_numpy(inp[key]).cuda() for key in ("q", "xt", "u"))
+    g = A.verify(zt, q, xt, u, w.T, w.top_p, w.k, workspace=ws)
+    torch.cuda.synchronize()
+    counters = ws[A.COUNTERS_OFFSET:A.COUNTERS_OFFSET + 64].view(torch.int32).cpu().numpy().tolist()
+    return {key: v.cpu().numpy() for key, v in g.items()}, counters
+
+
+def test_hints_carried_to_the_next_call_change_no_result(A, orc):
+    # 680 rows shaped like the 256000-id workload, twice on one workspace:
+    # the first call's first wave has no hints; the second call takes the
+    # first call's from the workspace, so all its rows are hinted and nearly
+    # all take the sketch-led pass.  Hints choose a pass only: the same bits, the
+    # oracle's results.  A workspace whose hint area holds another call's
+    # hints or noise gives the same bits too.
+    w = gen.make_workload(40, 16, 256000, "bf16", sigma=3.0, rho=0.9, T=0.6, top_p=0.8, k=128, seed=61)
+    inp = dict(gen.generate(w))
+    rows = w.B * (w.K + 1)
+    ws = torch.zeros(A.workspace_bytes(w.B, w.K, w.V, w.k), dtype=torch.uint8, device="cuda")
+    g1, c1 = _verify_ws(A, w, inp, ws)
+    g2, c2 = _verify_ws(A, w, inp, ws)
+    # (a few rows start while this call's own first rows say that fewer than
+    # 98% were short, and count instead)
+    assert c1[HINTED] < rows and c2[HINTED] == rows and c2[SKETCH_LED] >= rows - rows // 32, (c1, c2)
+    assert c2[SKETCH_LED] > c1[SKETCH_LED], (c1, c2)
+    for key in g1:
+        assert np.array_equal(g1[key], g2[key]), key
+    o = orc.verify(inp["z"], inp["q"], inp["xt"], inp["u"], w.T, w.top_p, w.k)
+    res = parity.compare_verify(inp, g2, o, w.top_p, True, w.k)
+    assert res["checked_seqs"] >= 32
+    # another call's hints (another top_p) and then noise in the hint area
+    w2 = gen.make_workload(40, 16, 256000, "bf16", sigma=3.0, rho=0.9, T=0.6, top_p=0.5, k=128, seed=61)
+    _verify_ws(A, w2, inp, ws)
+    g3, c3 = _verify_ws(A, w, inp, ws)
+    assert c3[HINTED] < rows, c3
+    ws[:256] = torch.randint(0, 256, (256,), dtype=torch.uint8, device="cuda")
+    g4, _ = _verify_ws(A, w, inp, ws)
+    for key in g1:
+        assert np.array_equal(g1[key], g3[key]) and np.array_equal(g1[key], g4[key]), key
+
+
 def test_sketch_led_row_with_a_long_nucleus_counts_again(A, orc):
     # The first 800 rows have four dominant ids (short nuclei), the last
     # 288 flat logits (nuclei of most of the row).  Rows that start after
