@@ -85,6 +85,17 @@ constexpr int CREC = 1536;          // recorded chunks (16-byte chunk + its inde
 constexpr int LCAP = 2048;          // listed ids, expanded from the records after the stream
 constexpr int WCAP = 2048;          // work area: ordered candidates
 constexpr int SMEM_F32 = CREC * 20 + LCAP * 8 + NBIN * 4;
+// float32 rows of a launch that fits one wave at two CTAs per SM take wider
+// areas (and a deeper first capture): more records and list entries per row
+template <int W>
+struct F32Caps {
+    static constexpr int CR = W == 2 ? 3584 : CREC;  // recorded chunks
+    static constexpr int LC = W == 2 ? 4096 : LCAP;  // listed ids
+    static constexpr int WC = W == 2 ? 4096 : WCAP;  // ordered candidates
+    static constexpr int MARGIN = W == 2 ? MARGIN_BINS + 2 : MARGIN_BINS;
+    static constexpr int SMEM = CR * 20 + LC * 8 + NBIN * 4;
+};
+
 constexpr int RANK_MAX = 512;       // ids ordered by direct ranking (more: bitonic sort)
 static_assert(WS_DEPTH + NSB <= WS_COUNTERS / 4, "the depth histogram fits the counters area");
 static_assert(4 * NUC_CAP * 8 <= SMEM_BF && 4 * NUC_CAP * 8 <= SMEM_F32, "the draw's scratch fits");
@@ -92,6 +103,9 @@ static_assert(GCAP * 4 <= HW * 4 && PCAP * 8 <= SKG * 2 && HW <= PCAP, "the alia
 static_assert(PCAP <= SK_TMP && GCAP * 4 <= (SK_EMASS - SK_TMP) * 8 && PCAP <= SK_EMASS - SK_TMP &&
                   SK_EMASS + HW <= SKG / 4, "the sketch-led areas fit");
 static_assert(WCAP * 8 <= CREC * 20 && RANK_MAX * 2 <= LCAP, "the float32 work areas fit");
+static_assert(F32Caps<2>::WC * 8 <= F32Caps<2>::CR * 20 && RANK_MAX * 2 <= F32Caps<2>::LC &&
+                  2 * (F32Caps<2>::SMEM + 1024) <= 228 * 1024,
+              "the wide float32 areas fit, two CTAs per SM");
 
 __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
     s = a + b;
@@ -302,8 +316,10 @@ __device__ __forceinline__ unsigned long long id_fx(float v, float c, float kref
     return to_fx(ex2(fmaf(v, c, -kref)));
 }
 
-template <int DT>
+template <int DT, int W>
 __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
+    constexpr int CREC = F32Caps<W>::CR, LCAP = F32Caps<W>::LC, WCAP = F32Caps<W>::WC;
+    constexpr int MARGIN_BINS = F32Caps<W>::MARGIN;
     using E = Elem<DT>;
     constexpr int EPC = E::EPC;
     constexpr bool BF = DT == ACES_BF16;
@@ -1571,9 +1587,9 @@ void rows_cap_layout(RowArgs &a, int dt) {
 
 // The dynamic shared memory above 48 KB needs an opt-in per device, set
 // once per device on the first launch there (outside any stream capture).
-template <int DT>
+template <int DT, int W>
 static cudaError_t launch_cap_dt(const RowArgs &a, cudaStream_t s) {
-    constexpr int smem = DT == ACES_BF16 ? SMEM_BF : SMEM_F32;
+    constexpr int smem = DT == ACES_BF16 ? SMEM_BF : F32Caps<W>::SMEM;
     static std::mutex mu;
     static bool ready[64];
     int dev = 0;
@@ -1581,18 +1597,20 @@ static cudaError_t launch_cap_dt(const RowArgs &a, cudaStream_t s) {
     {
         std::lock_guard<std::mutex> lock(mu);
         if (!ready[dev]) {
-            const cudaError_t e = cudaFuncSetAttribute(k_rows_cap<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+            const cudaError_t e = cudaFuncSetAttribute(k_rows_cap<DT, W>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
             if (e != cudaSuccess) return e;
             ready[dev] = true;
         }
     }
-    k_rows_cap<DT><<<(unsigned)a.rows, NTC, smem, s>>>(a);
+    k_rows_cap<DT, W><<<(unsigned)a.rows, NTC, smem, s>>>(a);
     return cudaGetLastError();
 }
 
 // one CTA per row (16-byte aligned rows)
 cudaError_t launch_rows_cap(const RowArgs &a, int dt, cudaStream_t s) {
-    return dt == ACES_BF16 ? launch_cap_dt<ACES_BF16>(a, s) : launch_cap_dt<ACES_F32>(a, s);
+    if (dt == ACES_BF16) return launch_cap_dt<ACES_BF16, 1>(a, s);
+    // (float32: the wide areas when the launch is one wave at two CTAs per SM)
+    return a.rows <= 2 * a.nsm ? launch_cap_dt<ACES_F32, 2>(a, s) : launch_cap_dt<ACES_F32, 1>(a, s);
 }
 
 #ifdef ACES_CHECKED

@@ -199,14 +199,15 @@ def test_bitonic_order_for_many_candidates(A, orc):
 
 
 def test_more_candidates_than_the_list_falls_back(A, orc):
-    # 3000 near-equal float32 ids: the capture exceeds the 2048-id list, so
-    # every row goes to the exact general kernel
-    V = 64000
+    # 5000 near-equal float32 ids, each in its own chunk: the capture
+    # exceeds the 3584 records of a one-wave launch (1536 in larger ones),
+    # so every row goes to the exact general kernel
+    V = 128000
     w = gen.make_workload(2, 1, V, "f32", T=1.0, top_p=0.8, k=32, seed=32)
     rng = np.random.default_rng(32)
     z = np.full((2, 2, V), -30.0, np.float32)
-    ids = np.arange(3000) * 21
-    z[:, :, ids] = rng.uniform(0.0, 0.5, size=(2, 2, 3000)).astype(np.float32)
+    ids = np.arange(5000) * 21
+    z[:, :, ids] = rng.uniform(0.0, 0.5, size=(2, 2, 5000)).astype(np.float32)
     counters, res = _run(A, orc, w, z)
     assert counters[FALLBACK] == 4, counters
     assert res["checked_seqs"] == 2
