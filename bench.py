@@ -162,10 +162,19 @@ KERNEL_SOURCES = {
 }
 
 
+def _code_only(text: str) -> str:
+    """The source without its comments and blank space (a change of comments
+    alone leaves the kernel, and so the captured counters, as they were)."""
+    import re
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
 def kernel_source_hash(kernel: str) -> str:
     h = hashlib.sha256()
     for f in KERNEL_SOURCES[kernel]:
-        h.update(open(os.path.join(ROOT, "paper_2609_02514_gb300", "csrc", f), "rb").read())
+        h.update(_code_only(open(os.path.join(ROOT, "paper_2609_02514_gb300", "csrc", f)).read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -14,34 +14,45 @@
 //             running max shared by the CTA's warps.
 //   depth     D bounds how far below the row max the nucleus crossing (top_p
 //             = 1: the payload's end) lies: a quantile of the depths that the
-//             call's finished rows published, plus a margin (before any has
-//             finished: NSB bins of T/4).  D only decides what is kept; every
-//             result below is proved from exact sums.
-//   keep      bfloat16: every id >= (running max - D) increments a shared-
-//             memory counter of its bfloat16 value (a window of HW values),
-//             and a sketch keeps the max of every group of 4 to 8 chunks;
+//             call's finished rows published, plus a margin (before 32 have
+//             finished: those the previous call on the same workspace left,
+//             for bfloat16 rows of the same shape; else NSB bins of T/4).  D
+//             only decides what is kept; every result below is proved from
+//             exact sums.
+//   keep      bfloat16, counting pass: every id >= (running max - D)
+//             increments a shared-memory counter of its bfloat16 value (a
+//             window of HW values); sketch-led pass (when nearly all finished
+//             rows had short nuclei): nothing is counted while streaming.
+//             Both keep the max of every group of 4 to 8 chunks in a sketch.
 //             float32: every 16-byte chunk holding an id >= the threshold is
 //             recorded (chunk and index).  The running max only rises, so at
-//             the end every id >= (row max - D) was kept.
+//             the end every id >= (row max - D) was kept (or, sketch-led,
+//             lies in a group whose max reaches it).
 //   finish    from the exact row max and exp-sum, exact 2^-40 fixed-point
-//             masses give the nucleus crossing (else the row goes to the exact
-//             general kernel):
-//             bfloat16  one warp scans the value counts for the crossing
-//                       value, the number j of its ids inside the nucleus and
-//                       the payload's last value; the sketch's groups whose
-//                       max reaches that value are re-read and their ids at or
-//                       above it ordered.  When the crossing value's ids are
-//                       among them the j-th (in id order) is the cut;
-//                       otherwise the row keeps (value, j) and the resolve
-//                       step finds that id only for the rows it draws from.
-//             float32   the recorded ids are binned by (m - z)/(T/8) with
-//                       exact masses; the bins up to the crossing bin are
-//                       ordered (direct ranking up to 512 ids, bitonic sort
-//                       above) and one warp finds the crossing.
+//             masses give the nucleus crossing (a crossing below the kept
+//             values: a second counting pass over the row; a capacity
+//             exceeded: the exact general kernel):
+//             bfloat16  (sketch-led: the groups reaching row max - D are read
+//                       back and their ids counted first) one warp scans the
+//                       value counts for the crossing value, the number j of
+//                       its ids inside the nucleus and the payload's last
+//                       value; the sketch's groups whose max reaches that
+//                       value are re-read and their ids at or above it
+//                       ordered.  When the crossing value's ids are among them
+//                       the j-th (in id order) is the cut; otherwise the row
+//                       keeps (value, j) and the resolve step finds that id
+//                       only for the rows it draws from.
+//             float32   the recorded ids are binned by (m - z)/(T/8); the bins
+//                       up to the one where a lower bound of the mass reaches
+//                       the target are ordered (direct ranking up to 512 ids,
+//                       else bin by bin with a rank inside each bin) and one
+//                       warp finds the crossing with exact prefix sums.
 //             Then the payload, the tail mass, the accept test of the draft
 //             token at this position and the per-row state; the CTA that
 //             finishes a sequence's last row draws its token when row pi's
 //             nucleus was kept.
+// On launches of four waves or more, the j-th CTA each SM starts with waits
+// j x 10 us first, so that the first wave's epilogues do not coincide.
 #include <climits>
 #include <mutex>
 #include <type_traits>
