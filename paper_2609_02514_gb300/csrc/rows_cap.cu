@@ -379,13 +379,11 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     const uint32_t NI = E::NEG_INF_WORD;
     const bool all_in = a.top_p >= 1.0f;
 
-    // the draft token of this position, fetched early by thread 0
+    // the draft token of this position, fetched early by thread 0 and kept
+    // in shared memory across the stream (xb, bq, iq are set after it)
     int xb = -1, bq = 0, iq = 0;
-    if (a.K > 0) {
-        bq = r / (a.K + 1);
-        iq = r % (a.K + 1);
-        if (tid == 0 && iq < a.K) xb = a.xt[(size_t)bq * a.K + iq];
-    }
+    int xb0 = -1;
+    if (a.K > 0 && tid == 0 && r % (a.K + 1) < a.K) xb0 = a.xt[(size_t)(r / (a.K + 1)) * a.K + r % (a.K + 1)];
     if (BF) {
         for (int i = tid; i < HW; i += NTC) hist[i] = 0u;
     } else {
@@ -527,6 +525,7 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
         }
     }
     publish_max(im);
+    if (tid == 0) s_xb = xb0;
     __syncthreads();
     const float m1 = running_max();  // the sample's max
     const bool have = m1 > -INFINITY && m1 < INFINITY;
@@ -548,6 +547,11 @@ __global__ void __launch_bounds__(NTC, 4) k_rows_cap(RowArgs a) {
     // reduces the row max, the reference and the exp-sum (fp32 two-sum tree,
     // fp64 in warp 0); true when the row is not a distribution (handled)
     auto finish_sums = [&]() -> bool {
+        if (a.K > 0) {
+            bq = r / (a.K + 1);
+            iq = r % (a.K + 1);
+        }
+        xb = tid == 0 ? s_xb : -1;
         if (xb >= 0 && xb < a.V) {
             zx = E::load1(row, xb);
             qx = __ldg(a.q + ((size_t)bq * a.K + iq) * a.V + xb);
