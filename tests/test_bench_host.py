@@ -58,3 +58,17 @@ def test_two_gloo_ranks_shard_sequences_and_take_the_max_time():
     assert set(gathered[0]).isdisjoint(gathered[1])
     assert first_u[0] != first_u[1]
     assert res[0][2] == res[1][2] == 2.5
+
+
+def test_traffic_figures_follow_the_kernel_code_not_its_comments():
+    # The bench reports a kernel's captured DRAM traffic only while the
+    # kernel's code is the code it was captured from: comments and spacing
+    # do not count, a changed statement does.
+    import sys
+    sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+    import bench
+    src = "int f(int x) {\n  // the square\n  return x * x; /* (exact) */\n}\n"
+    assert bench._code_only(src) == bench._code_only("int f(int x) {  return x * x;\n\n}")
+    assert bench._code_only(src) != bench._code_only(src.replace("x * x", "x + x"))
+    for k in bench.KERNEL_SOURCES:
+        assert len(bench.kernel_source_hash(k)) == 16
